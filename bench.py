@@ -1,0 +1,474 @@
+#!/usr/bin/env python3
+"""Benchmark of spliced decode attention on the Qwen3-8B-shaped donor-noise
+ladder sweep (36 layers, 32 q / 8 kv heads, d = 128, 32 prompts x 4096-token
+prompt span, 5 donor slots, 1024 decode steps, (L, W) grid 5 x 4, 512-sequence
+decode batches).
+
+One *step* = one decode step of one 512-sequence batch through all layers:
+per layer one ``suffix_kv_append`` and one ``spliced_decode_attn``.  Steps
+walk the decode steps t of the sweep in a stratified order (t_k at the
+midpoints of K equal slices of 1..T), so the mix of generated-span lengths and
+splice epochs matches the whole run.  The metric is sequence-steps per second
+(one sequence-step = all layers and heads of one sequence at one t).
+
+Legs (one JSON line on rank 0):
+* value: device-resident inputs, CUDA events around exactly K steps;
+* roofline: per-kernel launch durations from CUDA events recorded by the
+  library around each launch, over a second pass of the same K steps;
+  algorithmic bytes per launch from the descriptor's source maps;
+* e2e: the same K steps through the C ABI with the step's queries and new
+  K/V copied from pinned host memory and the outputs copied back, copies
+  overlapped with compute on separate streams;
+* cpu_baseline: the fp64 CPU oracle on a bounded sample of (sequence,
+  layer, step) units of the same batch, on the host's cores.
+``--impl reference`` times that oracle alone as the reference arm.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "spliced decode-attn sequence-steps/s (Qwen3-8B-shaped sweep); HBM GB/s vs peak"
+UNIT = "seq-steps/s"
+WORKLOAD = "qwen3-8b-ladder"
+NOMINAL_HBM_GBS = 8000.0
+
+
+def step_schedule(T: int, n: int, offset: int = 0):
+    """Decode steps at the midpoints of n equal slices of 1..T."""
+    return [1 + ((2 * ((k + offset) % n) + 1) * T) // (2 * n) for k in range(n)]
+
+
+def read_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as fh:
+            d = json.load(fh)
+        return float(d.get("hbm_gbs", 6800.0)), "measured"
+    return 6800.0, "fallback"
+
+
+# --------------------------------------------------------------------------
+# algorithmic bytes (what the method must move), from the source maps
+# --------------------------------------------------------------------------
+def algorithmic_bytes(sb, layer: int, step: int):
+    from paper_2605_30574_gb300 import splice as S
+    wl = sb.wl
+    st = S.splice_plan_stats(sb.desc, layer, step)
+    m = S.splice_debug_source_map(sb.desc, layer, step)
+    spans = {(sb.seqs[s].prompt, code) for s, code in enumerate(m) if code != S.SRC_ZERO}
+    n_read = sum(1 for code in m if code != S.SRC_ZERO)
+    kv_row = wl.num_kv_heads * wl.head_dim * 4          # K + V bf16 of one position, all kv heads
+    q_bytes = wl.num_q_heads * wl.head_dim * 2
+    return {
+        "prompt_span_pass": len(spans) * st["prompt_visible"] * kv_row + n_read * q_bytes,
+        "generated_span_pass": sb.B * st["suffix_visible"] * kv_row + sb.B * q_bytes,
+        "merge": sb.B * wl.num_q_heads * wl.head_dim * 4,
+        "append": sb.B * wl.num_kv_heads * wl.head_dim * 8 if step >= 1 else 0,
+    }
+
+
+# --------------------------------------------------------------------------
+# clocks during the timed region
+# --------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.fh, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.fh.close()
+
+    def summary(self):
+        if not self.path or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"]}
+        rows = []
+        with open(self.path) as fh:
+            for line in fh:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        pw = [float(r[3]) for r in rows if r[3].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        loaded = [x for x in sm if x > 0.5 * max(sm)] if sm else []
+        return {"sm_mhz": statistics.median(loaded) if loaded else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "power_w_max": max(pw) if pw else None,
+                "samples": len(rows), "reasons": reasons}
+
+
+# --------------------------------------------------------------------------
+# CPU oracle leg
+# --------------------------------------------------------------------------
+class _Provider:
+    """Pre-generated oracle inputs of one (sequence, layer, step) unit."""
+
+    def __init__(self, d):
+        self.d = d
+
+    def q(self, s, t, l):
+        return self.d["q"]
+
+    def clean_kv(self, p, l):
+        return self.d["clean"]
+
+    def donor_kv(self, p, k, l):
+        return self.d["donor"]
+
+    def suffix_kv(self, s, l, i0, i1):
+        return self.d["suffix"]
+
+
+def _make_unit_inputs(wl, s, l, t):
+    import oracle
+    from paper_2605_30574_gb300.synth import host as H
+    g = H.SynthInputs(wl)
+    seq = wl.sequences()[s]
+    src = oracle.splice_source(seq.L, seq.W, seq.slot, wl.slot_kinds[seq.slot], l, t)
+    d = {"q": g.q(s, t, l), "clean": g.clean_kv(seq.prompt, l), "suffix": g.suffix_kv(s, l, 0, t)}
+    d["donor"] = g.donor_kv(seq.prompt, seq.slot, l) if src >= oracle.SRC_DONOR0 else None
+    return seq, d
+
+
+def _oracle_worker(name, units, barrier, results):
+    import oracle
+    from paper_2605_30574_gb300.synth import workloads as W
+    wl = W.get(name)
+    prepared = [(s, l, t) + _make_unit_inputs(wl, s, l, t) for (s, l, t) in units]
+    barrier.wait()
+    t0 = time.perf_counter()
+    for s, l, t, seq, d in prepared:
+        oracle.decode_attn(wl, _Provider(d), s, seq, l, t)
+    results.put((len(prepared), time.perf_counter() - t0))
+
+
+def run_oracle_sample(name, units_per_core, cores, seed, batch=0):
+    """Times the oracle on cores x units_per_core units (generation excluded)."""
+    import multiprocessing as mp
+    from paper_2605_30574_gb300.synth import workloads as W
+    wl = W.get(name)
+    rng = np.random.default_rng(seed)
+    lo, hi = wl.batch_range(batch)
+    ts = step_schedule(wl.max_steps, 16)
+    units = [[(int(rng.integers(lo, hi)), int(rng.integers(0, wl.num_layers)), int(ts[rng.integers(0, 16)]))
+              for _ in range(units_per_core)] for _ in range(cores)]
+    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        os.environ[k] = "1"
+    ctx = mp.get_context("spawn")
+    barrier = ctx.Barrier(cores + 1)
+    results = ctx.Queue()
+    procs = [ctx.Process(target=_oracle_worker, args=(name, units[c], barrier, results)) for c in range(cores)]
+    for p in procs:
+        p.start()
+    barrier.wait()
+    t0 = time.perf_counter()
+    got = [results.get() for _ in procs]
+    wall = time.perf_counter() - t0
+    for p in procs:
+        p.join()
+    n_units = sum(g[0] for g in got)
+    return n_units, wall
+
+
+def cpu_baseline(name, budget_s=15.0):
+    from paper_2605_30574_gb300.synth import workloads as W
+    wl = W.get(name)
+    cores = max(1, min(os.cpu_count() or 1, 16))
+    # calibrate: one unit on one core
+    n1, w1 = run_oracle_sample(name, 1, 1, seed=99)
+    per_unit = w1 / max(n1, 1)
+    upc = int(max(1, min(64, budget_s / per_unit)))
+    n, wall = run_oracle_sample(name, upc, cores, seed=7)
+    value = n / wall / wl.num_layers
+    return {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": (f"{n} (sequence, layer, step) units of batch 0 ({upc} per core, random layer, steps at "
+                       f"16 stratified t), fp64 numpy oracle, input generation excluded; "
+                       f"{wall:.1f} s wall; seq-steps = units / {wl.num_layers} layers")}
+
+
+def reference_arm(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    from paper_2605_30574_gb300.synth import workloads as W
+    wl = W.get(args.workload)
+    cores = max(1, min(os.cpu_count() or 1, 16))
+    for w in range(args.warmup):
+        run_oracle_sample(args.workload, 1, cores, seed=1000 + w)
+    total_units, total_wall = 0, 0.0
+    for k in range(args.steps):
+        n, wall = run_oracle_sample(args.workload, 1, cores, seed=k)
+        total_units += n
+        total_wall += wall
+    value = total_units / total_wall / wl.num_layers
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * total_wall / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic",
+            "config": {"workload": describe(wl), "batch": wl.batch},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": f"each step: {cores} random (sequence, layer, step) units of batch 0, "
+                                       f"one per core; input generation excluded"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+def describe(wl):
+    return (f"{wl.name}: {wl.num_layers} layers, {wl.num_q_heads}/{wl.num_kv_heads} heads, d {wl.head_dim}, "
+            f"{wl.num_prompts} prompts x {wl.prompt_len}-token span, {len(wl.slot_kinds)} donor slots, "
+            f"T {wl.max_steps}, L {list(wl.L_values)} x W {list(wl.W_values)}, {wl.batch}-sequence batches")
+
+
+# --------------------------------------------------------------------------
+# GPU arm
+# --------------------------------------------------------------------------
+def gpu_arm(args):
+    import torch
+    import torch.distributed as dist
+    from paper_2605_30574_gb300 import build as B
+    from paper_2605_30574_gb300 import splice as S
+    from paper_2605_30574_gb300.sweep import SweepBatch
+    from paper_2605_30574_gb300.synth import device as SD
+    from paper_2605_30574_gb300.synth import workloads as W
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    B.build()
+    wl = W.get(args.workload)
+    batch = (args.batch + rank) % wl.num_batches()   # weak scaling: one sweep batch per GPU
+    sb = SweepBatch(wl, batch)
+    N = wl.num_layers
+    steps = step_schedule(wl.max_steps, args.steps)
+    warm = step_schedule(wl.max_steps, max(args.warmup, 1), offset=0)[: args.warmup]
+    dev = torch.device("cuda", local)
+    # this step's inputs for every layer, generated ahead (excluded from timing)
+    def gen(ts):
+        qs = torch.empty((len(ts), N) + tuple(sb.q.shape), dtype=torch.bfloat16, device=dev)
+        kn = torch.empty((len(ts), N) + tuple(sb.k_new.shape), dtype=torch.bfloat16, device=dev)
+        vn = torch.empty_like(kn)
+        for i, t in enumerate(ts):
+            for l in range(N):
+                SD.fill_q(wl, sb.s0, l, t, qs[i, l])
+                SD.fill_new_kv(wl, sb.s0, l, t, kn[i, l], vn[i, l])
+        return qs, kn, vn
+
+    qs, kn, vn = gen(steps)
+    wq, wkn, wvn = gen(warm) if warm else (None, None, None)
+    outs = torch.empty((N,) + tuple(sb.out.shape), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def run_step(t, q, k_new, v_new, out):
+        for l in range(N):
+            S.suffix_kv_append(sb.desc, l, t, k_new[l], v_new[l], sb.k_suffix, sb.v_suffix, stream)
+            S.spliced_decode_attn(sb.desc, l, t, q[l], sb.k_clean, sb.v_clean, sb.k_donor, sb.v_donor,
+                                  sb.k_suffix, sb.v_suffix, out[l], sb.ws, stream=stream)
+
+    for i, t in enumerate(warm):
+        run_step(t, wq[i], wkn[i], wvn[i], outs)
+    torch.cuda.synchronize()
+
+    # ---- value: exactly K steps, device-resident inputs ----
+    launches0 = S.splice_kernel_launches(sb.desc)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        ev0.record(stream)
+        for i, t in enumerate(steps):
+            run_step(t, qs[i], kn[i], vn[i], outs)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    ms = ev0.elapsed_time(ev1)
+    gpu_launches = S.splice_kernel_launches(sb.desc) - launches0
+    S.splice_check_device_error(sb.desc)
+
+    units = sb.B * len(steps)
+    if world > 1:
+        tt = torch.tensor([ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+        uu = torch.tensor([units], device=dev, dtype=torch.float64)
+        dist.all_reduce(uu)
+        units = int(uu.item())
+    value = units / (ms / 1000.0)
+
+    # ---- algorithmic bytes of the timed steps ----
+    per_kind = {"append": 0, "prompt_span_pass": 0, "generated_span_pass": 0, "merge": 0}
+    for t in steps:
+        for l in range(N):
+            for k, v in algorithmic_bytes(sb, l, t).items():
+                per_kind[k] += v
+    total_bytes = sum(per_kind.values())
+
+    # ---- roofline pass: per-launch events recorded by the library ----
+    S.splice_profile_enable(sb.desc, True)
+    S.splice_profile_read(sb.desc)
+    torch.cuda.synchronize()
+    for i, t in enumerate(steps):
+        run_step(t, qs[i], kn[i], vn[i], outs)
+    torch.cuda.synchronize()
+    prof = S.splice_profile_read(sb.desc)
+    S.splice_profile_enable(sb.desc, False)
+    peak, peak_kind = read_peaks()
+    dom = max(prof, key=lambda k: prof[k][1])
+    n_l, ms_l = prof[dom]
+    achieved = (per_kind[dom] / max(n_l, 1)) / ((ms_l / max(n_l, 1)) / 1000.0) / 1e9
+    kernels = {k: {"launches": v[0], "ms_total": round(v[1], 3), "share": round(v[1] / sum(x[1] for x in prof.values()), 4),
+                   "GBps": round(per_kind[k] / (v[1] / 1000.0) / 1e9, 1) if v[1] > 0 else None}
+               for k, v in prof.items()}
+
+    # ---- e2e: host buffers through the C ABI, copies overlapped ----
+    e2e = None
+    if not args.no_e2e:
+        e2e = e2e_leg(sb, steps, qs, kn, vn, run_step, dev)
+    del qs, kn, vn
+
+    if rank == 0:
+        cpu = None if args.no_cpu_baseline else cpu_baseline(args.workload)
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": len(steps),
+            "warmup": args.warmup, "ms_per_step": ms / len(steps), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": describe(wl), "batch": f"batch {batch} of {wl.num_batches()}: sequences "
+                                                           f"{sb.s0}-{sb.s0 + sb.B - 1}",
+                       "decode_steps_t": steps, "l2": "inputs larger than L2 (every step streams >10 GB); no flush",
+                       "parallelism": f"{world} GPU(s), one sweep batch each, no collective"},
+            "hbm": {"algorithmic_GB_per_step": round(total_bytes / len(steps) / 1e9, 3),
+                    "achieved_GBps": round(total_bytes / (ms / 1000.0) / 1e9 / max(world, 1) * max(world, 1), 1),
+                    "frac_of_measured": round(total_bytes / (ms / 1000.0) / 1e9 / peak, 4),
+                    "frac_of_8TBps": round(total_bytes / (ms / 1000.0) / 1e9 / NOMINAL_HBM_GBS, 4)},
+            "roofline": {"kernel": dom, "bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
+                         "unit": "GB/s", "frac": round(achieved / peak, 4), "peak_source": peak_kind,
+                         "traffic": None, "bytes_per_launch": per_kind[dom] // max(n_l, 1),
+                         "ms_per_launch": ms_l / max(n_l, 1)},
+            "kernels": kernels,
+            "e2e": e2e, "gpu_launches": gpu_launches, "clocks": clk.summary(), "cpu_baseline": cpu,
+        }
+        print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def e2e_leg(sb, steps, qs, kn, vn, run_step, dev):
+    import torch
+    K = len(steps)
+    N = sb.wl.num_layers
+    h_q = torch.empty(qs.shape, dtype=qs.dtype, pin_memory=True)
+    h_kn = torch.empty(kn.shape, dtype=kn.dtype, pin_memory=True)
+    h_vn = torch.empty(vn.shape, dtype=vn.dtype, pin_memory=True)
+    h_q.copy_(qs.cpu())
+    h_kn.copy_(kn.cpu())
+    h_vn.copy_(vn.cpu())
+    d_q = [torch.empty(qs.shape[1:], dtype=qs.dtype, device=dev) for _ in range(2)]
+    d_kn = [torch.empty(kn.shape[1:], dtype=kn.dtype, device=dev) for _ in range(2)]
+    d_vn = [torch.empty(vn.shape[1:], dtype=vn.dtype, device=dev) for _ in range(2)]
+    d_out = [torch.empty((N,) + tuple(sb.out.shape), dtype=torch.float32, device=dev) for _ in range(2)]
+    h_out = [torch.empty((N,) + tuple(sb.out.shape), dtype=torch.float32, pin_memory=True) for _ in range(2)]
+    comp = torch.cuda.current_stream()
+    h2d = torch.cuda.Stream()
+    d2h = torch.cuda.Stream()
+    in_ready = [torch.cuda.Event() for _ in range(K)]
+    comp_done = [torch.cuda.Event() for _ in range(K)]
+    out_free = [torch.cuda.Event() for _ in range(K)]
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(h2d)
+    for k, t in enumerate(steps):
+        b = k % 2
+        with torch.cuda.stream(h2d):
+            if k >= 2:
+                h2d.wait_event(comp_done[k - 2])          # slot b no longer read by compute
+            d_q[b].copy_(h_q[k], non_blocking=True)
+            d_kn[b].copy_(h_kn[k], non_blocking=True)
+            d_vn[b].copy_(h_vn[k], non_blocking=True)
+            in_ready[k].record(h2d)
+        comp.wait_event(in_ready[k])
+        if k >= 2:
+            comp.wait_event(out_free[k - 2])              # output slot b copied out
+        run_step(t, d_q[b], d_kn[b], d_vn[b], d_out[b])
+        comp_done[k].record(comp)
+        with torch.cuda.stream(d2h):
+            d2h.wait_event(comp_done[k])
+            h_out[b].copy_(d_out[b], non_blocking=True)
+            out_free[k].record(d2h)
+    e1.record(d2h)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    h2d_bytes = (qs[0].numel() + kn[0].numel() + vn[0].numel()) * 2
+    d2h_bytes = d_out[0].numel() * 4
+    return {"value": sb.B * K / (ms / 1000.0), "unit": UNIT, "h2d_bytes_per_step": int(h2d_bytes),
+            "d2h_bytes_per_step": int(d2h_bytes), "ms_per_step": ms / K,
+            "how": "pinned host queries + new K/V per step copied H2D, outputs of every layer copied D2H, "
+                   "on two copy streams overlapped with compute (double-buffered)"}
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=16)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=WORKLOAD)
+    ap.add_argument("--batch", type=int, default=0)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.impl == "reference":
+        return reference_arm(args)
+    return gpu_arm(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,514 @@
+// C ABI of the spliced decode-attention library (include/splice.h):
+// argument validation, descriptor lifetime, device tables, and the launch
+// sequence of one decode step.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "splice_internal.h"
+
+using splice::AttnParams;
+using splice::Plan;
+
+struct splice_desc {
+    bool on_device = false;
+    splice_model_shape shape{};
+    int P = 0, Tp = 0, Dslots = 0, Dst = 0, B = 0, T = 0;
+    std::vector<int32_t> slot_stored;   // [Dslots] stored-donor index or -1
+    std::vector<splice_seq> seqs;
+    Plan plan;
+    int device = -1;
+    // Device tables, one allocation.
+    char* dev = nullptr;
+    std::vector<char> staging;          // host image of `dev`, kept for the async upload
+    uint8_t* d_src = nullptr;
+    int32_t* d_seq_prompt = nullptr;
+    int32_t* d_seq_slot = nullptr;
+    int32_t* d_slot_stored = nullptr;
+    int32_t* d_tiles = nullptr;
+    int32_t* d_group_prompt = nullptr;
+    int32_t* d_group_src = nullptr;
+    int32_t* d_group_seqs = nullptr;
+    unsigned* d_err = nullptr;
+    // Measurement: launch counter and optional per-launch event timing.
+    long long launches = 0;
+    bool profiling = false;
+    std::vector<std::pair<cudaEvent_t, cudaEvent_t>> events[SPLICE_KERNEL_KINDS];
+    size_t events_used[SPLICE_KERNEL_KINDS] = {0, 0, 0, 0};
+};
+
+namespace {
+
+thread_local std::string g_last_error;
+
+splice_status fail(splice_status st, const char* f, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, f);
+    std::vsnprintf(buf, sizeof buf, f, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return st;
+}
+
+splice_status cuda_fail(cudaError_t e, const char* what) {
+    return fail(SPLICE_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Restores the caller's current device on scope exit.
+struct DeviceGuard {
+    int prev = -1;
+    bool changed = false;
+    cudaError_t err = cudaSuccess;
+    explicit DeviceGuard(int dev) {
+        err = cudaGetDevice(&prev);
+        if (err == cudaSuccess && prev != dev) {
+            err = cudaSetDevice(dev);
+            changed = err == cudaSuccess;
+        }
+    }
+    ~DeviceGuard() {
+        if (changed) cudaSetDevice(prev);
+    }
+};
+
+splice_status validate_create(const splice_model_shape* sh, int P, int Tp, int Dslots,
+                              const splice_donor_kind* kinds, int B, const splice_seq* seqs,
+                              int T, splice_desc** out) {
+    if (!out) return fail(SPLICE_EINVAL, "out is NULL");
+    *out = nullptr;
+    if (!sh) return fail(SPLICE_EINVAL, "shape is NULL");
+    if (sh->num_layers < 1) return fail(SPLICE_EINVAL, "num_layers %d < 1", sh->num_layers);
+    if (sh->num_kv_heads < 1 || sh->num_q_heads < sh->num_kv_heads ||
+        sh->num_q_heads % sh->num_kv_heads != 0)
+        return fail(SPLICE_EINVAL, "num_q_heads %d must be a positive multiple of num_kv_heads %d",
+                    sh->num_q_heads, sh->num_kv_heads);
+    if (sh->num_q_heads / sh->num_kv_heads > 16)
+        return fail(SPLICE_EINVAL, "group size %d > 16", sh->num_q_heads / sh->num_kv_heads);
+    if (sh->head_dim != 64 && sh->head_dim != 128 && sh->head_dim != 256)
+        return fail(SPLICE_EINVAL, "head_dim %d not in {64, 128, 256}", sh->head_dim);
+    if (sh->sliding_window < 0 || sh->global_every < 0)
+        return fail(SPLICE_EINVAL, "negative sliding_window or global_every");
+    if (!std::isfinite(sh->sm_scale)) return fail(SPLICE_EINVAL, "sm_scale is not finite");
+    if (P < 1 || Tp < 1 || B < 1 || T < 1)
+        return fail(SPLICE_EINVAL, "num_prompts, prompt_len, num_seqs and max_steps must be >= 1");
+    if (Dslots < 1 || Dslots > 250) return fail(SPLICE_EINVAL, "num_donor_slots %d not in [1, 250]", Dslots);
+    if (!kinds || !seqs) return fail(SPLICE_EINVAL, "slot_kinds or seqs is NULL");
+    int dst = 0;
+    for (int k = 0; k < Dslots; ++k) {
+        if (int(kinds[k]) < 0 || int(kinds[k]) > 4)
+            return fail(SPLICE_EINVAL, "slot %d has unknown donor kind %d", k, int(kinds[k]));
+        if (kinds[k] != SPLICE_DONOR_ZERO) ++dst;
+    }
+    for (int s = 0; s < B; ++s) {
+        const splice_seq& q = seqs[s];
+        if (q.prompt_id < 0 || q.prompt_id >= P)
+            return fail(SPLICE_EINVAL, "seq %d: prompt_id %d out of range", s, q.prompt_id);
+        if (q.donor_slot < 0 || q.donor_slot >= Dslots)
+            return fail(SPLICE_EINVAL, "seq %d: donor_slot %d out of range", s, q.donor_slot);
+        if (q.L < 0 || q.W < 0) return fail(SPLICE_EINVAL, "seq %d: negative L or W", s);
+    }
+    const long long rows = 1LL * P * sh->num_layers * sh->num_kv_heads * Tp;
+    if (rows >= (1LL << 31) || rows * std::max(dst, 1) >= (1LL << 31))
+        return fail(SPLICE_EINVAL, "prompt stores exceed 2^31 rows");
+    return SPLICE_OK;
+}
+
+splice_status create_common(const splice_model_shape* sh, int P, int Tp, int Dslots,
+                            const splice_donor_kind* kinds, int B, const splice_seq* seqs, int T,
+                            splice_desc** out, splice_desc*& d) {
+    splice_status st = validate_create(sh, P, Tp, Dslots, kinds, B, seqs, T, out);
+    if (st != SPLICE_OK) return st;
+    d = new (std::nothrow) splice_desc();
+    if (!d) return fail(SPLICE_ENOMEM, "descriptor allocation failed");
+    try {
+        d->shape = *sh;
+        d->P = P;
+        d->Tp = Tp;
+        d->Dslots = Dslots;
+        d->B = B;
+        d->T = T;
+        d->seqs.assign(seqs, seqs + B);
+        d->slot_stored.assign(Dslots, -1);
+        for (int k = 0; k < Dslots; ++k)
+            if (kinds[k] != SPLICE_DONOR_ZERO) d->slot_stored[k] = d->Dst++;
+        std::string e = splice::build_plan(*sh, P, Tp, Dslots, kinds, B, seqs, T, d->plan);
+        if (!e.empty()) {
+            delete d;
+            d = nullptr;
+            return fail(SPLICE_EINVAL, "%s", e.c_str());
+        }
+    } catch (const std::bad_alloc&) {
+        delete d;
+        d = nullptr;
+        return fail(SPLICE_ENOMEM, "host allocation failed while planning");
+    }
+    return SPLICE_OK;
+}
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Runs one kernel launcher, counting it and, when profiling, bracketing it
+// with a pair of events on its stream.
+template <class F>
+cudaError_t timed_launch(splice_desc* d, int kind, void* stream, F&& launch) {
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    std::pair<cudaEvent_t, cudaEvent_t>* ev = nullptr;
+    if (d->profiling) {
+        auto& pool = d->events[kind];
+        if (d->events_used[kind] == pool.size()) {
+            cudaEvent_t a, b;
+            cudaError_t e = cudaEventCreate(&a);
+            if (e != cudaSuccess) return e;
+            e = cudaEventCreate(&b);
+            if (e != cudaSuccess) {
+                cudaEventDestroy(a);
+                return e;
+            }
+            pool.emplace_back(a, b);
+        }
+        ev = &pool[d->events_used[kind]++];
+        cudaError_t e = cudaEventRecord(ev->first, st);
+        if (e != cudaSuccess) return e;
+    }
+    cudaError_t e = cudaError_t(launch());
+    if (e != cudaSuccess) return e;
+    ++d->launches;
+    if (ev) e = cudaEventRecord(ev->second, st);
+    return e;
+}
+
+size_t workspace_bytes_of(const splice_desc* d) {
+    const size_t rows = size_t(d->B) * d->shape.num_q_heads;
+    const size_t ml = align_up(size_t(splice::kMaxSplits) * rows * sizeof(float2), 256);
+    const size_t o = size_t(splice::kMaxSplits) * rows * d->shape.head_dim * sizeof(float);
+    return ml + o;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* splice_status_str(splice_status s) {
+    switch (s) {
+        case SPLICE_OK: return "ok";
+        case SPLICE_EINVAL: return "invalid argument";
+        case SPLICE_ENOMEM: return "out of memory";
+        case SPLICE_ECUDA: return "CUDA error";
+        case SPLICE_ESTATE: return "descriptor state does not allow this call";
+        case SPLICE_EDEVICE: return "kernel-side error";
+    }
+    return "unknown status";
+}
+
+const char* splice_last_error(void) { return g_last_error.c_str(); }
+
+splice_status splice_desc_create_host(const splice_model_shape* sh, int P, int Tp, int Dslots,
+                                       const splice_donor_kind* kinds, int B, const splice_seq* seqs,
+                                       int T, splice_desc** out) {
+    splice_desc* d = nullptr;
+    splice_status st = create_common(sh, P, Tp, Dslots, kinds, B, seqs, T, out, d);
+    if (st != SPLICE_OK) return st;
+    *out = d;
+    return SPLICE_OK;
+}
+
+splice_status splice_desc_create(const splice_model_shape* sh, int P, int Tp, int Dslots,
+                                  const splice_donor_kind* kinds, int B, const splice_seq* seqs,
+                                  int T, void* stream, splice_desc** out) {
+    splice_desc* d = nullptr;
+    splice_status st = create_common(sh, P, Tp, Dslots, kinds, B, seqs, T, out, d);
+    if (st != SPLICE_OK) return st;
+    cudaError_t e = cudaGetDevice(&d->device);
+    if (e != cudaSuccess) {
+        delete d;
+        return cuda_fail(e, "cudaGetDevice");
+    }
+    const Plan& pl = d->plan;
+    // Layout of the device table block.
+    struct Part {
+        const void* src;
+        size_t bytes;
+        size_t off;
+    };
+    std::vector<int32_t> seq_prompt(d->B), seq_slot(d->B);
+    for (int s = 0; s < d->B; ++s) {
+        seq_prompt[s] = d->seqs[s].prompt_id;
+        seq_slot[s] = d->seqs[s].donor_slot;
+    }
+    const unsigned zero = 0;
+    Part parts[] = {
+        {pl.src.data(), pl.src.size(), 0},
+        {seq_prompt.data(), seq_prompt.size() * 4, 0},
+        {seq_slot.data(), seq_slot.size() * 4, 0},
+        {d->slot_stored.data(), d->slot_stored.size() * 4, 0},
+        {pl.tiles.data(), pl.tiles.size() * 4, 0},
+        {pl.group_prompt.data(), pl.group_prompt.size() * 4, 0},
+        {pl.group_src.data(), pl.group_src.size() * 4, 0},
+        {pl.group_seqs.data(), pl.group_seqs.size() * 4, 0},
+        {&zero, sizeof zero, 0},
+    };
+    size_t total = 0;
+    for (Part& p : parts) {
+        p.off = total;
+        total = align_up(total + std::max<size_t>(p.bytes, 4), 256);
+    }
+    try {
+        d->staging.assign(total, 0);
+    } catch (const std::bad_alloc&) {
+        delete d;
+        return fail(SPLICE_ENOMEM, "host staging allocation failed");
+    }
+    for (const Part& p : parts)
+        if (p.bytes) std::memcpy(d->staging.data() + p.off, p.src, p.bytes);
+    e = cudaMalloc(reinterpret_cast<void**>(&d->dev), total);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        delete d;
+        return e == cudaErrorMemoryAllocation ? fail(SPLICE_ENOMEM, "cudaMalloc of %zu bytes failed", total)
+                                              : cuda_fail(e, "cudaMalloc");
+    }
+    e = cudaMemcpyAsync(d->dev, d->staging.data(), total, cudaMemcpyHostToDevice,
+                        static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) {
+        cudaFree(d->dev);
+        delete d;
+        return cuda_fail(e, "cudaMemcpyAsync of descriptor tables");
+    }
+    char* b = d->dev;
+    d->d_src = reinterpret_cast<uint8_t*>(b + parts[0].off);
+    d->d_seq_prompt = reinterpret_cast<int32_t*>(b + parts[1].off);
+    d->d_seq_slot = reinterpret_cast<int32_t*>(b + parts[2].off);
+    d->d_slot_stored = reinterpret_cast<int32_t*>(b + parts[3].off);
+    d->d_tiles = reinterpret_cast<int32_t*>(b + parts[4].off);
+    d->d_group_prompt = reinterpret_cast<int32_t*>(b + parts[5].off);
+    d->d_group_src = reinterpret_cast<int32_t*>(b + parts[6].off);
+    d->d_group_seqs = reinterpret_cast<int32_t*>(b + parts[7].off);
+    d->d_err = reinterpret_cast<unsigned*>(b + parts[8].off);
+    d->on_device = true;
+    *out = d;
+    return SPLICE_OK;
+}
+
+splice_status splice_desc_destroy(splice_desc* d) {
+    if (!d) return SPLICE_OK;
+    splice_status st = SPLICE_OK;
+    if (d->dev) {
+        DeviceGuard g(d->device);
+        for (auto& pool : d->events)
+            for (auto& ev : pool) {
+                cudaEventDestroy(ev.first);
+                cudaEventDestroy(ev.second);
+            }
+        cudaError_t e = cudaFree(d->dev);
+        if (e != cudaSuccess) st = cuda_fail(e, "cudaFree of descriptor tables");
+    }
+    delete d;
+    return st;
+}
+
+size_t splice_workspace_bytes(const splice_desc* d) { return d ? workspace_bytes_of(d) : 0; }
+
+int splice_num_stored_donor_slots(const splice_desc* d) { return d ? d->Dst : -1; }
+
+splice_status suffix_kv_append(splice_desc* d, int layer, int step, const splice_bf16* k_new,
+                               const splice_bf16* v_new, splice_bf16* k_suffix,
+                               splice_bf16* v_suffix, void* stream) {
+    if (!d) return fail(SPLICE_EINVAL, "descriptor is NULL");
+    if (!d->on_device) return fail(SPLICE_ESTATE, "host-only descriptor");
+    if (layer < 0 || layer >= d->shape.num_layers) return fail(SPLICE_EINVAL, "layer %d out of range", layer);
+    if (step < 1 || step > d->T) return fail(SPLICE_EINVAL, "append step %d not in [1, %d]", step, d->T);
+    if (!k_new || !v_new || !k_suffix || !v_suffix) return fail(SPLICE_EINVAL, "NULL tensor");
+    if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(k_suffix) || !aligned16(v_suffix))
+        return fail(SPLICE_EINVAL, "tensor not 16-byte aligned");
+    DeviceGuard g(d->device);
+    if (g.err != cudaSuccess) return cuda_fail(g.err, "cudaSetDevice");
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "earlier CUDA error");
+    e = timed_launch(d, 0, stream, [&] {
+        return splice::launch_append(k_new, v_new, k_suffix, v_suffix, d->B, d->shape.num_layers,
+                                     d->shape.num_kv_heads, d->shape.head_dim, d->T, layer, step, stream);
+    });
+    if (e != cudaSuccess) return cuda_fail(e, "append launch");
+    return SPLICE_OK;
+}
+
+splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const splice_bf16* q,
+                                  const splice_bf16* k_clean, const splice_bf16* v_clean,
+                                  const splice_bf16* k_donor, const splice_bf16* v_donor,
+                                  const splice_bf16* k_suffix, const splice_bf16* v_suffix, float* out,
+                                  void* workspace, size_t workspace_bytes, void* stream) {
+    if (!d) return fail(SPLICE_EINVAL, "descriptor is NULL");
+    if (!d->on_device) return fail(SPLICE_ESTATE, "host-only descriptor");
+    if (layer < 0 || layer >= d->shape.num_layers) return fail(SPLICE_EINVAL, "layer %d out of range", layer);
+    if (step < 0 || step > d->T) return fail(SPLICE_EINVAL, "step %d not in [0, %d]", step, d->T);
+    if (!q || !k_clean || !v_clean || !out || !workspace)
+        return fail(SPLICE_EINVAL, "NULL tensor or workspace");
+    if (step > 0 && (!k_suffix || !v_suffix)) return fail(SPLICE_EINVAL, "NULL generated-span store");
+    if (d->Dst > 0 && (!k_donor || !v_donor)) return fail(SPLICE_EINVAL, "NULL donor store");
+    const void* ptrs[] = {q, k_clean, v_clean, k_donor, v_donor, k_suffix, v_suffix, out, workspace};
+    for (const void* p : ptrs)
+        if (p && !aligned16(p)) return fail(SPLICE_EINVAL, "tensor not 16-byte aligned");
+    if (workspace_bytes < workspace_bytes_of(d))
+        return fail(SPLICE_EINVAL, "workspace of %zu bytes < %zu", workspace_bytes, workspace_bytes_of(d));
+    DeviceGuard g(d->device);
+    if (g.err != cudaSuccess) return cuda_fail(g.err, "cudaSetDevice");
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "earlier CUDA error");
+
+    const splice_model_shape& sh = d->shape;
+    const int tab = d->plan.table_of(layer, step);
+    const splice::Visible vis = splice::visible_keys(sh, d->Tp, layer, step);
+    const size_t rows = size_t(d->B) * sh.num_q_heads;
+    AttnParams p{};
+    p.q = q;
+    p.kc = k_clean;
+    p.vc = v_clean;
+    p.kd = k_donor;
+    p.vd = v_donor;
+    p.ks = k_suffix;
+    p.vs = v_suffix;
+    p.out = out;
+    p.ws_ml = static_cast<float2*>(workspace);
+    p.ws_o = reinterpret_cast<float*>(static_cast<char*>(workspace) +
+                                      align_up(size_t(splice::kMaxSplits) * rows * sizeof(float2), 256));
+    p.src = d->d_src + size_t(tab) * d->B;
+    p.seq_prompt = d->d_seq_prompt;
+    p.seq_slot = d->d_seq_slot;
+    p.slot_stored = d->d_slot_stored;
+    p.tiles = d->d_tiles + 4 * size_t(d->plan.table_tile_off[tab]);
+    p.n_tiles = d->plan.table_tile_off[tab + 1] - d->plan.table_tile_off[tab];
+    p.group_prompt = d->d_group_prompt;
+    p.group_src = d->d_group_src;
+    p.group_seqs = d->d_group_seqs;
+    p.err = d->d_err;
+    p.B = d->B;
+    p.N = sh.num_layers;
+    p.Hq = sh.num_q_heads;
+    p.Hkv = sh.num_kv_heads;
+    p.D = sh.head_dim;
+    p.G = sh.num_q_heads / sh.num_kv_heads;
+    p.Tp = d->Tp;
+    p.T = d->T;
+    p.Dst = d->Dst;
+    p.layer = layer;
+    p.step = step;
+    p.p_lo = vis.p_lo;
+    p.p_hi = vis.p_hi;
+    p.s_lo = vis.s_lo;
+    p.s_hi = vis.s_hi;
+    const int p_vis = vis.p_hi - vis.p_lo, s_vis = vis.s_hi - vis.s_lo;
+    auto splits = [](int n, int per, int cap) { return n <= 0 ? 0 : std::min(cap, (n + per - 1) / per); };
+    p.nsp = splits(p_vis, 512, splice::kMaxPrefixSplits);
+    p.nss = splits(s_vis, 512, splice::kMaxSuffixSplits);
+    p.p_chunk = p.nsp ? (p_vis + p.nsp - 1) / p.nsp : 0;
+    p.s_chunk = p.nss ? (s_vis + p.nss - 1) / p.nss : 0;
+    p.scale_log2 = sh.sm_scale * 1.4426950408889634f;
+
+    if (p.nsp) {
+        e = timed_launch(d, 1, stream, [&] { return splice::launch_partials_cc(p, true, stream); });
+        if (e != cudaSuccess) return cuda_fail(e, "prompt-span partials launch");
+    }
+    if (p.nss) {
+        e = timed_launch(d, 2, stream, [&] { return splice::launch_partials_cc(p, false, stream); });
+        if (e != cudaSuccess) return cuda_fail(e, "generated-span partials launch");
+    }
+    e = timed_launch(d, 3, stream, [&] { return splice::launch_merge(p, stream); });
+    if (e != cudaSuccess) return cuda_fail(e, "merge launch");
+    return SPLICE_OK;
+}
+
+splice_status splice_debug_source_map(splice_desc* d, int layer, int step, uint8_t* host_out) {
+    if (!d || !host_out) return fail(SPLICE_EINVAL, "NULL descriptor or output");
+    if (layer < 0 || layer >= d->shape.num_layers) return fail(SPLICE_EINVAL, "layer %d out of range", layer);
+    if (step < 0 || step > d->T) return fail(SPLICE_EINVAL, "step %d not in [0, %d]", step, d->T);
+    const int tab = d->plan.table_of(layer, step);
+    if (!d->on_device) {
+        std::memcpy(host_out, d->plan.src.data() + size_t(tab) * d->B, d->B);
+        return SPLICE_OK;
+    }
+    DeviceGuard g(d->device);
+    if (g.err != cudaSuccess) return cuda_fail(g.err, "cudaSetDevice");
+    cudaError_t e = cudaMemcpy(host_out, d->d_src + size_t(tab) * d->B, d->B, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy of the source map");
+    return SPLICE_OK;
+}
+
+splice_status splice_plan_stats(const splice_desc* d, int layer, int step, int* num_groups, int* num_tiles,
+                                int* prompt_visible, int* suffix_visible) {
+    if (!d) return fail(SPLICE_EINVAL, "NULL descriptor");
+    if (layer < 0 || layer >= d->shape.num_layers) return fail(SPLICE_EINVAL, "layer %d out of range", layer);
+    if (step < 0 || step > d->T) return fail(SPLICE_EINVAL, "step %d not in [0, %d]", step, d->T);
+    const int tab = d->plan.table_of(layer, step);
+    const splice::Visible v = splice::visible_keys(d->shape, d->Tp, layer, step);
+    if (num_groups) *num_groups = d->plan.table_group_off[tab + 1] - d->plan.table_group_off[tab];
+    if (num_tiles) *num_tiles = d->plan.table_tile_off[tab + 1] - d->plan.table_tile_off[tab];
+    if (prompt_visible) *prompt_visible = v.p_hi - v.p_lo;
+    if (suffix_visible) *suffix_visible = v.s_hi - v.s_lo;
+    return SPLICE_OK;
+}
+
+splice_status splice_check_device_error(splice_desc* d) {
+    if (!d) return fail(SPLICE_EINVAL, "NULL descriptor");
+    if (!d->on_device) return fail(SPLICE_ESTATE, "host-only descriptor");
+    DeviceGuard g(d->device);
+    if (g.err != cudaSuccess) return cuda_fail(g.err, "cudaSetDevice");
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
+    unsigned flag = 0;
+    e = cudaMemcpy(&flag, d->d_err, sizeof flag, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy of the error flag");
+    if (flag) {
+        const unsigned zero = 0;
+        cudaMemcpy(d->d_err, &zero, sizeof zero, cudaMemcpyHostToDevice);
+        return fail(SPLICE_EDEVICE, "kernel recorded error code 0x%x", flag);
+    }
+    return SPLICE_OK;
+}
+
+long long splice_kernel_launches(const splice_desc* d) { return d ? d->launches : -1; }
+
+splice_status splice_profile_enable(splice_desc* d, int enable) {
+    if (!d) return fail(SPLICE_EINVAL, "NULL descriptor");
+    if (!d->on_device) return fail(SPLICE_ESTATE, "host-only descriptor");
+    d->profiling = enable != 0;
+    return SPLICE_OK;
+}
+
+splice_status splice_profile_read(splice_desc* d, long long* launches, double* total_ms) {
+    if (!d) return fail(SPLICE_EINVAL, "NULL descriptor");
+    if (!d->on_device) return fail(SPLICE_ESTATE, "host-only descriptor");
+    DeviceGuard g(d->device);
+    if (g.err != cudaSuccess) return cuda_fail(g.err, "cudaSetDevice");
+    for (int k = 0; k < SPLICE_KERNEL_KINDS; ++k) {
+        double ms = 0.0;
+        for (size_t i = 0; i < d->events_used[k]; ++i) {
+            cudaError_t e = cudaEventSynchronize(d->events[k][i].second);
+            if (e != cudaSuccess) return cuda_fail(e, "cudaEventSynchronize");
+            float f = 0.f;
+            e = cudaEventElapsedTime(&f, d->events[k][i].first, d->events[k][i].second);
+            if (e != cudaSuccess) return cuda_fail(e, "cudaEventElapsedTime");
+            ms += f;
+        }
+        if (launches) launches[k] = (long long)d->events_used[k];
+        if (total_ms) total_ms[k] = ms;
+        d->events_used[k] = 0;
+    }
+    return SPLICE_OK;
+}
+
+const char* splice_kernel_kind_name(int kind) {
+    static const char* names[SPLICE_KERNEL_KINDS] = {"append", "prompt_span_pass", "generated_span_pass", "merge"};
+    return kind >= 0 && kind < SPLICE_KERNEL_KINDS ? names[kind] : "unknown";
+}
+
+}  // extern "C"

@@ -1,0 +1,97 @@
+// Internal declarations of the spliced decode-attention library (not part of
+// the C ABI).  Host planner types, kernel parameter blocks and launchers.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <string>
+#include <vector>
+
+#include <vector_types.h>
+
+#include "../../include/splice.h"
+
+namespace splice {
+
+// Largest number of key splits per row for the prompt span and for the
+// generated span; the workspace holds kMaxSplits partial states per row.
+constexpr int kMaxPrefixSplits = 8;
+constexpr int kMaxSuffixSplits = 8;
+constexpr int kMaxSplits = kMaxPrefixSplits + kMaxSuffixSplits;
+// Rows of one tensor-core prefix tile (tcgen05 M).
+constexpr int kTileRows = 128;
+
+// Host-side resolution of the splice rule (§3, Algorithm 1) into tables.
+//
+// Epoch e covers steps [epoch_bounds[e], epoch_bounds[e+1]) where the bounds
+// are 0 and every distinct W <= max_steps; layer class c covers layers
+// [class_bounds[c], class_bounds[c+1]) with bounds 0 and every distinct
+// L < N.  Within one (epoch, class) pair every sequence reads one source.
+struct Plan {
+    std::vector<int> epoch_bounds;
+    std::vector<int> class_bounds;
+    int num_tables = 0;                  // epochs * classes
+    std::vector<uint8_t> src;            // [num_tables][B] source codes
+    // (prompt, source) groups of the sequences that read a stored span.
+    std::vector<int32_t> table_group_off;   // [num_tables + 1]
+    std::vector<int32_t> group_prompt;      // [groups]
+    std::vector<int32_t> group_src;         // [groups] source code (CLEAN or DONOR0 + slot)
+    std::vector<int32_t> group_first;       // [groups] offset into group_seqs
+    std::vector<int32_t> group_count;       // [groups]
+    std::vector<int32_t> group_seqs;        // concatenated sequence indices
+    // Row tiles of at most kTileRows rows (seqs_per_tile sequences x G heads).
+    std::vector<int32_t> table_tile_off;    // [num_tables + 1]
+    std::vector<int32_t> tiles;             // [tiles][4]: group, first, count, 0
+    int seqs_per_tile = 0;
+
+    int table_of(int layer, int step) const;
+};
+
+std::string build_plan(const splice_model_shape& shape, int num_prompts, int prompt_len,
+                       int num_donor_slots, const splice_donor_kind* kinds, int num_seqs,
+                       const splice_seq* seqs, int max_steps, Plan& plan);
+
+// Visible key ranges of the step-t query at layer l: prompt positions
+// [p_lo, prompt_len) and generated entries [s_lo, step).
+struct Visible {
+    int p_lo, p_hi, s_lo, s_hi;
+};
+Visible visible_keys(const splice_model_shape& shape, int prompt_len, int layer, int step);
+
+// Parameter block of the attention kernels.
+struct AttnParams {
+    const uint16_t* q;
+    const uint16_t* kc;
+    const uint16_t* vc;
+    const uint16_t* kd;
+    const uint16_t* vd;
+    const uint16_t* ks;
+    const uint16_t* vs;
+    float* out;
+    float2* ws_ml;          // [kMaxSplits][B * Hq] (m in log2 units, l)
+    float* ws_o;            // [kMaxSplits][B * Hq][D]
+    const uint8_t* src;     // [B] source code of every sequence at this (layer, step)
+    const int32_t* seq_prompt;
+    const int32_t* slot_stored;   // [num_slots] stored-donor index or -1
+    const int32_t* seq_slot;      // [B]
+    const int32_t* tiles;         // tcgen05 prefix: [n_tiles][4] for this table
+    const int32_t* group_prompt;
+    const int32_t* group_src;
+    const int32_t* group_seqs;
+    unsigned* err;
+    int B, N, Hq, Hkv, D, G, Tp, T, Dst;
+    int layer, step;
+    int p_lo, p_hi, s_lo, s_hi;
+    int nsp, nss;                 // splits of the prompt span / generated span
+    int p_chunk, s_chunk;         // keys per split
+    int n_tiles;
+    float scale_log2;             // sm_scale * log2(e)
+};
+
+// Launchers (return the cudaError_t of the launch as int).
+int launch_append(const uint16_t* kn, const uint16_t* vn, uint16_t* ks, uint16_t* vs, int B,
+                  int N, int Hkv, int D, int T, int layer, int step, void* stream);
+int launch_partials_cc(const AttnParams& p, bool prefix, void* stream);
+int launch_merge(const AttnParams& p, void* stream);
+
+}  // namespace splice

@@ -1,0 +1,224 @@
+"""Thin ctypes binding of the C ABI in ``include/splice.h``.
+
+Argument marshalling only: tensors (torch tensors or raw integer device
+pointers) become pointers, the stream defaults to torch's current stream, and
+a non-OK status raises :class:`SpliceError`.  Every step of the path runs in
+``libsplice.so``; if the library is not built this module raises instead of
+falling back to anything else.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+_LIB = None
+_PKG = os.path.dirname(os.path.abspath(__file__))
+
+OK, EINVAL, ENOMEM, ECUDA, ESTATE, EDEVICE = range(6)
+DONOR_ZERO, DONOR_BLANK, DONOR_SAME_ALGO, DONOR_DIFF_ALGO, DONOR_DIFF_FAMILY = range(5)
+SRC_CLEAN, SRC_ZERO, SRC_DONOR0 = 0, 1, 2
+
+# Every function the C ABI exports, with its ctypes signature.
+_c_int, _c_size, _vp = ctypes.c_int, ctypes.c_size_t, ctypes.c_void_p
+
+
+class SpliceError(RuntimeError):
+    def __init__(self, status: int, where: str, detail: str):
+        super().__init__(f"{where}: status {status}: {detail}")
+        self.status = status
+
+
+class ModelShape(ctypes.Structure):
+    _fields_ = [("num_layers", ctypes.c_int), ("num_q_heads", ctypes.c_int),
+                ("num_kv_heads", ctypes.c_int), ("head_dim", ctypes.c_int),
+                ("sliding_window", ctypes.c_int), ("global_every", ctypes.c_int),
+                ("sm_scale", ctypes.c_float)]
+
+
+class Seq(ctypes.Structure):
+    _fields_ = [("prompt_id", ctypes.c_int), ("donor_slot", ctypes.c_int),
+                ("L", ctypes.c_int), ("W", ctypes.c_int)]
+
+
+SIGNATURES = {
+    "splice_desc_create": (_c_int, [ctypes.POINTER(ModelShape), _c_int, _c_int, _c_int,
+                                     ctypes.POINTER(ctypes.c_int), _c_int, ctypes.POINTER(Seq),
+                                     _c_int, _vp, ctypes.POINTER(_vp)]),
+    "splice_desc_create_host": (_c_int, [ctypes.POINTER(ModelShape), _c_int, _c_int, _c_int,
+                                          ctypes.POINTER(ctypes.c_int), _c_int, ctypes.POINTER(Seq),
+                                          _c_int, ctypes.POINTER(_vp)]),
+    "splice_desc_destroy": (_c_int, [_vp]),
+    "splice_workspace_bytes": (_c_size, [_vp]),
+    "splice_num_stored_donor_slots": (_c_int, [_vp]),
+    "suffix_kv_append": (_c_int, [_vp, _c_int, _c_int, _vp, _vp, _vp, _vp, _vp]),
+    "spliced_decode_attn": (_c_int, [_vp, _c_int, _c_int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                     _vp, _c_size, _vp]),
+    "splice_debug_source_map": (_c_int, [_vp, _c_int, _c_int, ctypes.POINTER(ctypes.c_uint8)]),
+    "splice_plan_stats": (_c_int, [_vp, _c_int, _c_int, ctypes.POINTER(_c_int), ctypes.POINTER(_c_int),
+                                   ctypes.POINTER(_c_int), ctypes.POINTER(_c_int)]),
+    "splice_check_device_error": (_c_int, [_vp]),
+    "splice_kernel_launches": (ctypes.c_longlong, [_vp]),
+    "splice_profile_enable": (_c_int, [_vp, _c_int]),
+    "splice_profile_read": (_c_int, [_vp, ctypes.POINTER(ctypes.c_longlong), ctypes.POINTER(ctypes.c_double)]),
+    "splice_kernel_kind_name": (ctypes.c_char_p, [_c_int]),
+    "splice_status_str": (ctypes.c_char_p, [_c_int]),
+    "splice_last_error": (ctypes.c_char_p, []),
+}
+
+
+def lib_path() -> str:
+    return os.path.join(_PKG, "libsplice.so")
+
+
+def lib() -> ctypes.CDLL:
+    global _LIB
+    if _LIB is None:
+        path = lib_path()
+        if not os.path.exists(path):
+            raise RuntimeError(f"{path} is not built: run paper_2605_30574_gb300.build.build() "
+                               "(there is no fallback path)")
+        L = ctypes.CDLL(path)
+        for name, (res, args) in SIGNATURES.items():
+            f = getattr(L, name)
+            f.restype = res
+            f.argtypes = args
+        _LIB = L
+    return _LIB
+
+
+def _check(status: int, where: str):
+    if status != OK:
+        detail = lib().splice_last_error().decode(errors="replace")
+        raise SpliceError(status, where, detail)
+
+
+def _ptr(x):
+    """Device pointer of a torch tensor (must be contiguous), an int, or None."""
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    if not x.is_contiguous():
+        raise ValueError("tensors passed to the splice library must be contiguous")
+    return x.data_ptr()
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+class Desc:
+    """Owns a ``splice_desc*``; destroyed on ``close()`` or garbage collection."""
+
+    def __init__(self, handle: int, num_seqs: int, on_device: bool):
+        self.handle = handle
+        self.num_seqs = num_seqs
+        self.on_device = on_device
+
+    def close(self):
+        if self.handle:
+            h, self.handle = self.handle, None
+            _check(lib().splice_desc_destroy(h), "splice_desc_destroy")
+
+    def __del__(self):
+        try:
+            if self.handle:
+                lib().splice_desc_destroy(self.handle)
+        except Exception:
+            pass
+
+
+def _marshal(shape, slot_kinds, seqs):
+    sh = ModelShape(**shape) if isinstance(shape, dict) else shape
+    kinds = (ctypes.c_int * len(slot_kinds))(*[int(k) for k in slot_kinds])
+    arr = (Seq * len(seqs))(*[Seq(int(s[0]), int(s[1]), int(s[2]), int(s[3])) for s in seqs])
+    return sh, kinds, arr
+
+
+def splice_desc_create(shape, num_prompts, prompt_len, slot_kinds, seqs, max_steps, stream=None) -> Desc:
+    """``seqs``: iterable of (prompt_id, donor_slot, L, W)."""
+    seqs = list(seqs)
+    sh, kinds, arr = _marshal(shape, slot_kinds, seqs)
+    out = _vp()
+    _check(lib().splice_desc_create(ctypes.byref(sh), num_prompts, prompt_len, len(slot_kinds), kinds,
+                                    len(seqs), arr, max_steps, _stream(stream), ctypes.byref(out)),
+           "splice_desc_create")
+    return Desc(out.value, len(seqs), True)
+
+
+def splice_desc_create_host(shape, num_prompts, prompt_len, slot_kinds, seqs, max_steps) -> Desc:
+    seqs = list(seqs)
+    sh, kinds, arr = _marshal(shape, slot_kinds, seqs)
+    out = _vp()
+    _check(lib().splice_desc_create_host(ctypes.byref(sh), num_prompts, prompt_len, len(slot_kinds), kinds,
+                                         len(seqs), arr, max_steps, ctypes.byref(out)),
+           "splice_desc_create_host")
+    return Desc(out.value, len(seqs), False)
+
+
+def splice_workspace_bytes(desc: Desc) -> int:
+    return int(lib().splice_workspace_bytes(desc.handle))
+
+
+def splice_num_stored_donor_slots(desc: Desc) -> int:
+    return int(lib().splice_num_stored_donor_slots(desc.handle))
+
+
+def suffix_kv_append(desc: Desc, layer, step, k_new, v_new, k_suffix, v_suffix, stream=None):
+    _check(lib().suffix_kv_append(desc.handle, layer, step, _ptr(k_new), _ptr(v_new), _ptr(k_suffix),
+                                  _ptr(v_suffix), _stream(stream)), "suffix_kv_append")
+
+
+def spliced_decode_attn(desc: Desc, layer, step, q, k_clean, v_clean, k_donor, v_donor, k_suffix, v_suffix,
+                        out, workspace, workspace_bytes=None, stream=None):
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    _check(lib().spliced_decode_attn(desc.handle, layer, step, _ptr(q), _ptr(k_clean), _ptr(v_clean),
+                                     _ptr(k_donor), _ptr(v_donor), _ptr(k_suffix), _ptr(v_suffix), _ptr(out),
+                                     _ptr(workspace), workspace_bytes, _stream(stream)),
+           "spliced_decode_attn")
+
+
+def splice_debug_source_map(desc: Desc, layer, step) -> bytes:
+    buf = (ctypes.c_uint8 * desc.num_seqs)()
+    _check(lib().splice_debug_source_map(desc.handle, layer, step, buf), "splice_debug_source_map")
+    return bytes(buf)
+
+
+def splice_plan_stats(desc: Desc, layer, step) -> dict:
+    g, t, p, s = ctypes.c_int(), ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
+    _check(lib().splice_plan_stats(desc.handle, layer, step, ctypes.byref(g), ctypes.byref(t),
+                                   ctypes.byref(p), ctypes.byref(s)), "splice_plan_stats")
+    return {"num_groups": g.value, "num_tiles": t.value, "prompt_visible": p.value, "suffix_visible": s.value}
+
+
+def splice_check_device_error(desc: Desc):
+    _check(lib().splice_check_device_error(desc.handle), "splice_check_device_error")
+
+
+KERNEL_KINDS = 4
+
+
+def splice_kernel_launches(desc: Desc) -> int:
+    return int(lib().splice_kernel_launches(desc.handle))
+
+
+def splice_profile_enable(desc: Desc, enable: bool = True):
+    _check(lib().splice_profile_enable(desc.handle, 1 if enable else 0), "splice_profile_enable")
+
+
+def splice_profile_read(desc: Desc) -> dict:
+    """{kind name: (launches, total ms)} since the previous read."""
+    n = (ctypes.c_longlong * KERNEL_KINDS)()
+    ms = (ctypes.c_double * KERNEL_KINDS)()
+    _check(lib().splice_profile_read(desc.handle, n, ms), "splice_profile_read")
+    return {lib().splice_kernel_kind_name(k).decode(): (int(n[k]), float(ms[k])) for k in range(KERNEL_KINDS)}
+
+
+def splice_status_str(status: int) -> str:
+    return lib().splice_status_str(status).decode()
