@@ -188,6 +188,41 @@ splice_status spliced_decode_attn(splice_desc* desc, int layer, int step, const 
                                   void* stream);
 
 /*
+ * spliced_decode_attn_static -- spliced_decode_attn for callers that cannot
+ * allocate device memory.  The paper has no counterpart; this is a
+ * deployment convenience.
+ *
+ * Some callers may not call cudaMalloc themselves: for example a plugin
+ * inside a host runtime that owns every device allocation through its own
+ * memory pool and hands the plugin only the tensors of the call, or a
+ * latency-critical decode loop in which an allocation (which can synchronise
+ * the device) is not acceptable.  Such a caller passes the same inputs and
+ * output as to spliced_decode_attn but no workspace: the partial softmax
+ * states live in a file-scope device array of SPLICE_STATIC_SCRATCH_BYTES
+ * (64 MiB) inside the library, which every GPU that loads the library holds
+ * until the process exits.  This call allocates nothing.
+ *
+ *   - The first call on a device looks up that array's device address (with
+ *     the tensors' device made current); make that first call before any
+ *     stream capture.
+ *   - A descriptor whose splice_workspace_bytes() exceeds
+ *     SPLICE_STATIC_SCRATCH_BYTES is rejected with SPLICE_EINVAL (reduce the
+ *     batch, or use spliced_decode_attn with a workspace).
+ *   - Every call on a device shares the one array, and it keeps the last
+ *     call's contents; nothing in it needs to start at zero.  Calls that
+ *     overlap on the GPU (other streams, other host threads, other
+ *     descriptors) race on it: serialise them.
+ *
+ * Arguments, layouts and errors are otherwise those of spliced_decode_attn.
+ */
+#define SPLICE_STATIC_SCRATCH_BYTES (64u << 20)
+splice_status spliced_decode_attn_static(splice_desc* desc, int layer, int step, const splice_bf16* q,
+                                         const splice_bf16* k_clean, const splice_bf16* v_clean,
+                                         const splice_bf16* k_donor, const splice_bf16* v_donor,
+                                         const splice_bf16* k_suffix, const splice_bf16* v_suffix,
+                                         float* out, void* stream);
+
+/*
  * splice_debug_source_map -- the prompt-span source every sequence reads at
  * (layer, step): host_out[s] = SPLICE_SRC_CLEAN, SPLICE_SRC_ZERO or
  * SPLICE_SRC_DONOR0 + slot.  For a device descriptor the map is read back

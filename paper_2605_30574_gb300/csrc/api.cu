@@ -196,6 +196,8 @@ size_t workspace_bytes_of(const splice_desc* d) {
 
 }  // namespace
 
+void splice::set_last_error(const char* msg) { g_last_error = msg; }
+
 extern "C" {
 
 const char* splice_status_str(splice_status s) {

@@ -88,6 +88,9 @@ struct AttnParams {
     float scale_log2;             // sm_scale * log2(e)
 };
 
+// Records the one-line reason splice_last_error() reports on this thread.
+void set_last_error(const char* msg);
+
 // Launchers (return the cudaError_t of the launch as int).
 int launch_append(const uint16_t* kn, const uint16_t* vn, uint16_t* ks, uint16_t* vs, int B,
                   int N, int Hkv, int D, int T, int layer, int step, void* stream);

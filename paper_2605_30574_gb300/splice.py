@@ -53,6 +53,8 @@ SIGNATURES = {
     "suffix_kv_append": (_c_int, [_vp, _c_int, _c_int, _vp, _vp, _vp, _vp, _vp]),
     "spliced_decode_attn": (_c_int, [_vp, _c_int, _c_int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
                                      _vp, _c_size, _vp]),
+    "spliced_decode_attn_static": (_c_int, [_vp, _c_int, _c_int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                            _vp]),
     "splice_debug_source_map": (_c_int, [_vp, _c_int, _c_int, ctypes.POINTER(ctypes.c_uint8)]),
     "splice_plan_stats": (_c_int, [_vp, _c_int, _c_int, ctypes.POINTER(_c_int), ctypes.POINTER(_c_int),
                                    ctypes.POINTER(_c_int), ctypes.POINTER(_c_int)]),
@@ -182,6 +184,19 @@ def spliced_decode_attn(desc: Desc, layer, step, q, k_clean, v_clean, k_donor, v
                                      _ptr(k_donor), _ptr(v_donor), _ptr(k_suffix), _ptr(v_suffix), _ptr(out),
                                      _ptr(workspace), workspace_bytes, _stream(stream)),
            "spliced_decode_attn")
+
+
+STATIC_SCRATCH_BYTES = 64 << 20
+
+
+def spliced_decode_attn_static(desc: Desc, layer, step, q, k_clean, v_clean, k_donor, v_donor, k_suffix,
+                               v_suffix, out, stream=None):
+    """spliced_decode_attn without a workspace: the library's static device
+    scratch holds the partial states (for callers that cannot allocate)."""
+    _check(lib().spliced_decode_attn_static(desc.handle, layer, step, _ptr(q), _ptr(k_clean), _ptr(v_clean),
+                                            _ptr(k_donor), _ptr(v_donor), _ptr(k_suffix), _ptr(v_suffix),
+                                            _ptr(out), _stream(stream)),
+           "spliced_decode_attn_static")
 
 
 def splice_debug_source_map(desc: Desc, layer, step) -> bytes:
