@@ -42,6 +42,10 @@ struct splice_desc {
     bool profiling = false;
     std::vector<std::pair<cudaEvent_t, cudaEvent_t>> events[SPLICE_KERNEL_KINDS];
     size_t events_used[SPLICE_KERNEL_KINDS] = {0, 0, 0, 0};
+    // TMA tensor maps of the clean and donor stores (K, V), rebuilt when the
+    // store pointers change.
+    alignas(64) unsigned char maps[4][128] = {};
+    const void* map_ptr[4] = {nullptr, nullptr, nullptr, nullptr};
 };
 
 namespace {
@@ -410,15 +414,30 @@ splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const spl
     p.s_hi = vis.s_hi;
     const int p_vis = vis.p_hi - vis.p_lo, s_vis = vis.s_hi - vis.s_lo;
     auto splits = [](int n, int per, int cap) { return n <= 0 ? 0 : std::min(cap, (n + per - 1) / per); };
-    p.nsp = splits(p_vis, 512, splice::kMaxPrefixSplits);
+    int tc_split = 0, tc_keys = 0;
+    if (p_vis > 0) tc_keys = splice::prefix_tc_split_keys(sh.head_dim, p_vis, &tc_split);
+    p.nsp = tc_split;
     p.nss = splits(s_vis, 512, splice::kMaxSuffixSplits);
-    p.p_chunk = p.nsp ? (p_vis + p.nsp - 1) / p.nsp : 0;
+    p.p_chunk = tc_keys;
     p.s_chunk = p.nss ? (s_vis + p.nss - 1) / p.nss : 0;
     p.scale_log2 = sh.sm_scale * 1.4426950408889634f;
 
-    if (p.nsp) {
-        e = timed_launch(d, 1, stream, [&] { return splice::launch_partials_cc(p, true, stream); });
-        if (e != cudaSuccess) return cuda_fail(e, "prompt-span partials launch");
+    if (p.nsp && p.n_tiles > 0) {
+        // Tensor maps over the stores viewed as [rows][d].
+        const long rows_c = long(d->P) * sh.num_layers * sh.num_kv_heads * d->Tp;
+        const void* ptrs[4] = {k_clean, v_clean, d->Dst ? k_donor : k_clean, d->Dst ? v_donor : v_clean};
+        const long rows[4] = {rows_c, rows_c, d->Dst ? rows_c * d->Dst : rows_c, d->Dst ? rows_c * d->Dst : rows_c};
+        const int box = splice::prefix_tc_box_rows(sh.head_dim);
+        for (int i = 0; i < 4; ++i) {
+            if (d->map_ptr[i] == ptrs[i]) continue;
+            if (splice::make_kv_tensor_map(d->maps[i], ptrs[i], rows[i], sh.head_dim, box) != 0)
+                return fail(SPLICE_ECUDA, "cuTensorMapEncodeTiled failed for store %d", i);
+            d->map_ptr[i] = ptrs[i];
+        }
+        e = timed_launch(d, 1, stream, [&] {
+            return splice::launch_prefix_tc(p, d->maps, tc_split, tc_keys, stream);
+        });
+        if (e != cudaSuccess) return cuda_fail(e, "prompt-span tensor-core pass launch");
     }
     if (p.nss) {
         e = timed_launch(d, 2, stream, [&] { return splice::launch_partials_cc(p, false, stream); });

@@ -97,4 +97,10 @@ int launch_append(const uint16_t* kn, const uint16_t* vn, uint16_t* ks, uint16_t
 int launch_partials_cc(const AttnParams& p, bool prefix, void* stream);
 int launch_merge(const AttnParams& p, void* stream);
 
+// Tensor-core prompt-span pass.  A tensor map is a 128-byte CUtensorMap.
+int make_kv_tensor_map(void* out_map, const void* base, long rows, int d, int box_rows);
+int prefix_tc_box_rows(int d);
+int prefix_tc_split_keys(int d, int p_vis, int* nsplit);
+int launch_prefix_tc(const AttnParams& p, const void* maps, int nsplit, int split_keys, void* stream);
+
 }  // namespace splice
