@@ -413,11 +413,21 @@ splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const spl
     p.s_lo = vis.s_lo;
     p.s_hi = vis.s_hi;
     const int p_vis = vis.p_hi - vis.p_lo, s_vis = vis.s_hi - vis.s_lo;
-    auto splits = [](int n, int per, int cap) { return n <= 0 ? 0 : std::min(cap, (n + per - 1) / per); };
     int tc_split = 0, tc_keys = 0;
     if (p_vis > 0) tc_keys = splice::prefix_tc_split_keys(sh.head_dim, p_vis, &tc_split);
     p.nsp = tc_split;
-    p.nss = splits(s_vis, 512, splice::kMaxSuffixSplits);
+    {
+        // Generated-span items: (sequence, kv head, row chunk, key split).
+        // Split so every resident warp gets about four items, but keep at
+        // least 64 keys per split.
+        const int G = sh.num_q_heads / sh.num_kv_heads;
+        const int gt = G % 4 == 0 ? 4 : (G % 2 == 0 ? 2 : 1);
+        const long base_items = long(d->B) * sh.num_kv_heads * (G / gt);
+        const long want = 4L * splice::generated_span_resident_warps(sh.head_dim);
+        int ns = int(std::min<long>(splice::kMaxSuffixSplits, std::max<long>(1, (want + base_items - 1) / base_items)));
+        ns = std::min(ns, std::max(1, s_vis / 64));
+        p.nss = s_vis > 0 ? ns : 0;
+    }
     p.p_chunk = tc_keys;
     p.s_chunk = p.nss ? (s_vis + p.nss - 1) / p.nss : 0;
     p.scale_log2 = sh.sm_scale * 1.4426950408889634f;
@@ -440,7 +450,7 @@ splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const spl
         if (e != cudaSuccess) return cuda_fail(e, "prompt-span tensor-core pass launch");
     }
     if (p.nss) {
-        e = timed_launch(d, 2, stream, [&] { return splice::launch_partials_cc(p, false, stream); });
+        e = timed_launch(d, 2, stream, [&] { return splice::launch_generated_span(p, stream); });
         if (e != cudaSuccess) return cuda_fail(e, "generated-span partials launch");
     }
     e = timed_launch(d, 3, stream, [&] { return splice::launch_merge(p, stream); });

@@ -1,0 +1,401 @@
+// Generated-span pass (CUDA cores): attention of the G query rows of one
+// (sequence, kv head) over that sequence's own generated-span K/V (§3: the
+// decode step attends over the prompt span and the t generated entries).
+//
+// HBM-bound streaming kernel:
+//   * persistent warps, each walking a fixed stream of work items
+//     (sequence, kv head, row chunk, key split) and, inside an item, blocks
+//     of 16 keys;
+//   * every block's K and V rows (contiguous in the generated-span store) are
+//     fetched by one bulk async copy (cp.async.bulk, mbarrier-tracked) into a
+//     two-stage per-warp ring; the next block -- of this item or the next one
+//     -- is in flight while the current one is computed;
+//   * a key row of d values is split over LPK = d / 16 lanes (16 dims each,
+//     two 16-byte chunks); q . k partial sums are reduced across the LPK
+//     lanes through a small shared-memory transpose (each lane ends with a
+//     few full logits), then probabilities are shared back the same way;
+//   * packed fp32x2 FMAs (FFMA2) for both q . k and p . v;
+//   * online softmax with a lazily moved reference max: the common path
+//     needs no rescale and no cross-lane max.
+// Emits the partial state (m, l, o) of every row, like the prompt-span pass.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+
+#include "splice_internal.h"
+#include "tc_ptx.cuh"
+
+namespace splice {
+namespace {
+
+constexpr unsigned kFull = 0xffffffffu;
+constexpr float kTau = 8.0f;
+constexpr unsigned kErrWaitGs = 0x10;
+
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// bf16 pair word -> (even dim, odd dim) as fp32
+__device__ __forceinline__ float2 unpack2(uint32_t w) {
+    return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
+}
+
+__device__ __forceinline__ void bulk_copy(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                 "l"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+
+template <int D, int GT>
+struct GS {
+    static constexpr int LPK = D / 16;              // lanes per key
+    static constexpr int KPW = 32 / LPK;            // key groups per warp
+    static constexpr int BK = 16;                   // keys per block
+    static constexpr int U = BK / KPW;              // keys per group per block
+    static constexpr int NV = U * GT;               // logits per group per block
+    static constexpr int VPL = NV >= LPK ? NV / LPK : 1;   // logits reduced by each lane
+    static constexpr int WARPS = D == 256 ? 2 : 4;
+    static constexpr int RED = NV + 4;              // padded floats per lane in the reduce buffer
+    static constexpr uint32_t ROW = D * 2;          // bytes of one key row
+    static constexpr uint32_t STAGE = BK * ROW * 2; // K + V block
+    // per-warp shared memory: 2 stages, reduce buffer, probability pairs, 2 barriers
+    static constexpr uint32_t OFF_RED = 2 * STAGE;
+    static constexpr uint32_t OFF_PP = OFF_RED + 32 * RED * 4;
+    static constexpr uint32_t OFF_BAR = OFF_PP + KPW * NV * 8;
+    static constexpr uint32_t PER_WARP = (OFF_BAR + 16 + 127) / 128 * 128;
+    static constexpr uint32_t SMEM = WARPS * PER_WARP;
+    static_assert(NV % 4 == 0 || NV < 4, "reduce layout");
+};
+
+// Where the keys of one work item live.
+struct Item {
+    const uint16_t* k;
+    const uint16_t* v;
+    int s, h, rc, split, k0, k1, nblk;
+};
+
+template <int D, int GT>
+__device__ __forceinline__ bool item_at(const AttnParams& P, int idx, int n_items, Item& it) {
+    if (idx >= n_items) return false;
+    const int n_rc = P.G / GT;
+    int rem = idx;
+    it.split = rem % P.nss;
+    rem /= P.nss;
+    it.rc = rem % n_rc;
+    rem /= n_rc;
+    it.h = rem % P.Hkv;
+    it.s = rem / P.Hkv;
+    const size_t blk = ((size_t(it.s) * P.N + P.layer) * P.Hkv + it.h) * size_t(P.T);
+    it.k = P.ks + blk * D;
+    it.v = P.vs + blk * D;
+    it.k0 = P.s_lo + it.split * P.s_chunk;
+    it.k1 = min(P.s_hi, it.k0 + P.s_chunk);
+    it.nblk = it.k1 > it.k0 ? (it.k1 - it.k0 + 15) / 16 : 0;
+    return true;
+}
+
+template <int D, int GT>
+__global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
+    gs_kernel(const AttnParams P, int n_items) {
+    using C = GS<D, GT>;
+    extern __shared__ __align__(128) uint8_t smem[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    uint8_t* ws = smem + warp * C::PER_WARP;
+    const uint32_t wbase = tc::smem_u32(ws);
+    const uint32_t bar0 = wbase + C::OFF_BAR;
+    float* red = reinterpret_cast<float*>(ws + C::OFF_RED);
+    float2* pp = reinterpret_cast<float2*>(ws + C::OFF_PP);
+
+    const int gi = lane / C::LPK, dl = lane % C::LPK;
+    const int c0 = dl, c1 = dl + C::LPK;
+    const int gwarp = blockIdx.x * C::WARPS + warp;
+    const int nwarps = gridDim.x * C::WARPS;
+    volatile int abort_flag = 0;
+
+    if (lane == 0) {
+        tc::mbar_init(bar0, 1);
+        tc::mbar_init(bar0 + 8, 1);
+        tc::fence_mbar_init();
+    }
+    __syncwarp();
+
+    // ---- issue cursor: walks (item, block) units of this warp's stream ----
+    Item iss;
+    int iss_idx = gwarp, iss_b = 0;
+    bool iss_ok = item_at<D, GT>(P, iss_idx, n_items, iss);
+    while (iss_ok && iss.nblk == 0) {
+        iss_idx += nwarps;
+        iss_ok = item_at<D, GT>(P, iss_idx, n_items, iss);
+    }
+    int issued = 0;
+    auto issue_next = [&]() {
+        if (!iss_ok) return;
+        const int stg = issued & 1;
+        const int j = iss.k0 + iss_b * 16;
+        const int nk = min(16, iss.k1 - j);
+        const uint32_t bytes = uint32_t(nk) * C::ROW;
+        if (lane == 0) {
+            const uint32_t dst = wbase + stg * C::STAGE;
+            tc::mbar_arrive_expect_tx(bar0 + 8 * stg, 2 * bytes);
+            bulk_copy(dst, iss.k + size_t(j) * D, bytes, bar0 + 8 * stg);
+            bulk_copy(dst + C::BK * C::ROW, iss.v + size_t(j) * D, bytes, bar0 + 8 * stg);
+        }
+        ++issued;
+        if (++iss_b >= iss.nblk) {
+            iss_b = 0;
+            do {
+                iss_idx += nwarps;
+                iss_ok = item_at<D, GT>(P, iss_idx, n_items, iss);
+            } while (iss_ok && iss.nblk == 0);
+        }
+    };
+    issue_next();
+    issue_next();
+
+    int consumed = 0;
+    bool ok = true;
+    Item it;
+    for (int idx = gwarp; ok && item_at<D, GT>(P, idx, n_items, it); idx += nwarps) {
+        // q rows of this item, pre-scaled into log2 units, as dim pairs
+        float2 q2[GT][8];
+#pragma unroll
+        for (int g = 0; g < GT; ++g) {
+            const int hq = it.h * P.G + it.rc * GT + g;
+            const uint4* qr = reinterpret_cast<const uint4*>(P.q + (size_t(it.s) * P.Hq + hq) * D);
+            const uint4 a = qr[c0], b = qr[c1];
+            const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const float2 f = unpack2(w[i]);
+                q2[g][i] = make_float2(f.x * P.scale_log2, f.y * P.scale_log2);
+            }
+        }
+        float m[GT], l[GT];
+        float2 o2[GT][8];
+#pragma unroll
+        for (int g = 0; g < GT; ++g) {
+            m[g] = -INFINITY;
+            l[g] = 0.f;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) o2[g][i] = make_float2(0.f, 0.f);
+        }
+
+        for (int b = 0; b < it.nblk; ++b) {
+            const int stg = consumed & 1;
+            const bool got = tc::mbar_wait(bar0 + 8 * stg, uint32_t(consumed >> 1) & 1u, &abort_flag, P.err, kErrWaitGs);
+            if (!__all_sync(kFull, got)) {
+                ok = false;
+                break;
+            }
+            const uint8_t* kst = ws + stg * C::STAGE;
+            const uint8_t* vst = kst + C::BK * C::ROW;
+            const int jb = it.k0 + b * 16;
+
+            // ---- partial q . k over this lane's 16 dims ----
+            float dot[C::NV];
+#pragma unroll
+            for (int u = 0; u < C::U; ++u) {
+                const int kb = u * C::KPW + gi;
+                const uint4 ka = *reinterpret_cast<const uint4*>(kst + kb * C::ROW + c0 * 16);
+                const uint4 kc = *reinterpret_cast<const uint4*>(kst + kb * C::ROW + c1 * 16);
+                const uint32_t w[8] = {ka.x, ka.y, ka.z, ka.w, kc.x, kc.y, kc.z, kc.w};
+                float2 k2[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) k2[i] = unpack2(w[i]);
+#pragma unroll
+                for (int g = 0; g < GT; ++g) {
+                    float2 acc = __fmul2_rn(q2[g][0], k2[0]);
+#pragma unroll
+                    for (int i = 1; i < 8; ++i) acc = __ffma2_rn(q2[g][i], k2[i], acc);
+                    dot[u * GT + g] = acc.x + acc.y;
+                }
+            }
+            // ---- transpose-reduce across the LPK lanes of the group ----
+            float* myred = red + lane * C::RED;
+            if constexpr (C::NV % 4 == 0) {
+#pragma unroll
+                for (int v = 0; v < C::NV; v += 4)
+                    *reinterpret_cast<float4*>(myred + v) = make_float4(dot[v], dot[v + 1], dot[v + 2], dot[v + 3]);
+            } else {
+#pragma unroll
+                for (int v = 0; v < C::NV; ++v) myred[v] = dot[v];
+            }
+            __syncwarp();
+            float sv[C::VPL];
+            int gv[C::VPL];
+            bool need = false;
+#pragma unroll
+            for (int i = 0; i < C::VPL; ++i) {
+                const int v = (dl * C::VPL + i) % C::NV;
+                float acc = 0.f;
+#pragma unroll
+                for (int q = 0; q < C::LPK; ++q) acc += red[(gi * C::LPK + q) * C::RED + v];
+                const int u = v / GT;
+                gv[i] = v % GT;
+                const bool valid = jb + u * C::KPW + gi < it.k1;
+                sv[i] = valid ? acc : -INFINITY;
+                need |= sv[i] > m[gv[i]] + kTau;
+            }
+            if (__any_sync(kFull, need)) {
+                // rare: some row's reference max moves; share every logit of
+                // the group and recompute the per-row block maxima
+                __syncwarp();
+#pragma unroll
+                for (int i = 0; i < C::VPL; ++i) red[(gi * C::LPK) * C::RED + (dl * C::VPL + i) % C::NV] = sv[i];
+                __syncwarp();
+#pragma unroll
+                for (int g = 0; g < GT; ++g) {
+                    float mb = -INFINITY;
+#pragma unroll
+                    for (int u = 0; u < C::U; ++u) mb = fmaxf(mb, red[(gi * C::LPK) * C::RED + u * GT + g]);
+                    if (mb > m[g] + kTau) {
+                        const float alpha = ex2(m[g] - mb);
+                        l[g] *= alpha;
+                        const float2 a2 = make_float2(alpha, alpha);
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) o2[g][i] = __fmul2_rn(o2[g][i], a2);
+                        m[g] = mb;
+                    }
+                }
+            }
+            // ---- probabilities, shared back as (p, p) pairs ----
+            __syncwarp();
+            float2* mypp = pp + gi * C::NV;
+#pragma unroll
+            for (int i = 0; i < C::VPL; ++i) {
+                const float mg = m[gv[i]] == -INFINITY ? 0.f : m[gv[i]];
+                const float p = ex2(sv[i] - mg);
+                if (C::NV >= C::LPK || dl < C::NV) mypp[(dl * C::VPL + i) % C::NV] = make_float2(p, p);
+            }
+            __syncwarp();
+            float2 p2[C::NV];
+#pragma unroll
+            for (int v = 0; v < C::NV; v += 2) {
+                const float4 t = *reinterpret_cast<const float4*>(mypp + v);
+                p2[v] = make_float2(t.x, t.y);
+                if (v + 1 < C::NV) p2[v + 1] = make_float2(t.z, t.w);
+            }
+#pragma unroll
+            for (int u = 0; u < C::U; ++u) {
+#pragma unroll
+                for (int g = 0; g < GT; ++g) l[g] += p2[u * GT + g].x;
+            }
+            // ---- o += p . v over this lane's 16 dims ----
+#pragma unroll
+            for (int u = 0; u < C::U; ++u) {
+                const int kb = u * C::KPW + gi;
+                if (jb + kb < it.k1) {
+                    const uint4 va = *reinterpret_cast<const uint4*>(vst + kb * C::ROW + c0 * 16);
+                    const uint4 vc = *reinterpret_cast<const uint4*>(vst + kb * C::ROW + c1 * 16);
+                    const uint32_t w[8] = {va.x, va.y, va.z, va.w, vc.x, vc.y, vc.z, vc.w};
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const float2 v2 = unpack2(w[i]);
+#pragma unroll
+                        for (int g = 0; g < GT; ++g) o2[g][i] = __ffma2_rn(p2[u * GT + g], v2, o2[g][i]);
+                    }
+                }
+            }
+            // stage free: every lane is done reading it
+            __syncwarp();
+            tc::fence_proxy_async_smem();
+            ++consumed;
+            issue_next();
+        }
+        if (!ok) break;
+
+        // ---- combine the KPW key groups of the warp, write the partial ----
+#pragma unroll
+        for (int off = C::LPK; off < 32; off <<= 1) {
+#pragma unroll
+            for (int g = 0; g < GT; ++g) {
+                const float mo = __shfl_xor_sync(kFull, m[g], off);
+                const float lo = __shfl_xor_sync(kFull, l[g], off);
+                const float M = fmaxf(m[g], mo);
+                const float a = m[g] == -INFINITY ? 0.f : ex2(m[g] - M);
+                const float bb = mo == -INFINITY ? 0.f : ex2(mo - M);
+                l[g] = l[g] * a + lo * bb;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const float ox = __shfl_xor_sync(kFull, o2[g][i].x, off);
+                    const float oy = __shfl_xor_sync(kFull, o2[g][i].y, off);
+                    o2[g][i] = make_float2(o2[g][i].x * a + ox * bb, o2[g][i].y * a + oy * bb);
+                }
+                m[g] = M;
+            }
+        }
+        if (gi == 0) {
+            const int slot = kMaxPrefixSplits + it.split;
+#pragma unroll
+            for (int g = 0; g < GT; ++g) {
+                const size_t row = size_t(it.s) * P.Hq + it.h * P.G + it.rc * GT + g;
+                const size_t idx2 = size_t(slot) * P.B * P.Hq + row;
+                float4* op = reinterpret_cast<float4*>(P.ws_o + idx2 * D);
+                op[2 * c0] = make_float4(o2[g][0].x, o2[g][0].y, o2[g][1].x, o2[g][1].y);
+                op[2 * c0 + 1] = make_float4(o2[g][2].x, o2[g][2].y, o2[g][3].x, o2[g][3].y);
+                op[2 * c1] = make_float4(o2[g][4].x, o2[g][4].y, o2[g][5].x, o2[g][5].y);
+                op[2 * c1 + 1] = make_float4(o2[g][6].x, o2[g][6].y, o2[g][7].x, o2[g][7].y);
+                if (dl == 0) P.ws_ml[idx2] = make_float2(m[g], l[g]);
+            }
+        }
+    }
+    // Copies still in flight (only after an abort) must land before exit.
+    for (; consumed < issued; ++consumed) {
+        volatile int no_abort = 0;
+        tc::mbar_wait(bar0 + 8 * (consumed & 1), uint32_t(consumed >> 1) & 1u, &no_abort, P.err, kErrWaitGs);
+    }
+}
+
+template <int D, int GT>
+int launch_gs_t(const AttnParams& p, int n_items, cudaStream_t st) {
+    using C = GS<D, GT>;
+    static int blocks_per_sm = 0, sms = 0;
+    if (!blocks_per_sm) {
+        cudaFuncSetAttribute(gs_kernel<D, GT>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks_per_sm, gs_kernel<D, GT>, C::WARPS * 32, C::SMEM);
+        if (blocks_per_sm < 1) blocks_per_sm = 1;
+    }
+    const long want = (long(n_items) + C::WARPS - 1) / C::WARPS;
+    const long cap = long(blocks_per_sm) * sms;
+    const unsigned grid = unsigned(want < cap ? want : cap);
+    gs_kernel<D, GT><<<grid, C::WARPS * 32, C::SMEM, st>>>(p, n_items);
+    return int(cudaGetLastError());
+}
+
+}  // namespace
+
+int generated_span_resident_warps(int d) {
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    // two 4-warp CTAs per SM (d <= 128), three 2-warp CTAs per SM (d = 256)
+    return sms * (d == 256 ? 6 : 8);
+}
+
+int launch_generated_span(const AttnParams& p, void* stream) {
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const int gt = p.G % 4 == 0 ? 4 : (p.G % 2 == 0 ? 2 : 1);
+    const long n_items = long(p.B) * p.Hkv * (p.G / gt) * p.nss;
+    if (n_items == 0) return 0;
+    switch (p.D * 8 + gt) {
+        case 64 * 8 + 1: return launch_gs_t<64, 1>(p, int(n_items), st);
+        case 64 * 8 + 2: return launch_gs_t<64, 2>(p, int(n_items), st);
+        case 64 * 8 + 4: return launch_gs_t<64, 4>(p, int(n_items), st);
+        case 128 * 8 + 1: return launch_gs_t<128, 1>(p, int(n_items), st);
+        case 128 * 8 + 2: return launch_gs_t<128, 2>(p, int(n_items), st);
+        case 128 * 8 + 4: return launch_gs_t<128, 4>(p, int(n_items), st);
+        case 256 * 8 + 1: return launch_gs_t<256, 1>(p, int(n_items), st);
+        case 256 * 8 + 2: return launch_gs_t<256, 2>(p, int(n_items), st);
+        case 256 * 8 + 4: return launch_gs_t<256, 4>(p, int(n_items), st);
+        default: return int(cudaErrorInvalidValue);
+    }
+}
+
+}  // namespace splice

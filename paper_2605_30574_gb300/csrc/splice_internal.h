@@ -94,7 +94,8 @@ void set_last_error(const char* msg);
 // Launchers (return the cudaError_t of the launch as int).
 int launch_append(const uint16_t* kn, const uint16_t* vn, uint16_t* ks, uint16_t* vs, int B,
                   int N, int Hkv, int D, int T, int layer, int step, void* stream);
-int launch_partials_cc(const AttnParams& p, bool prefix, void* stream);
+int launch_generated_span(const AttnParams& p, void* stream);
+int generated_span_resident_warps(int d);
 int launch_merge(const AttnParams& p, void* stream);
 
 // Tensor-core prompt-span pass.  A tensor map is a 128-byte CUtensorMap.
