@@ -44,11 +44,33 @@ METRIC = "spliced decode-attn sequence-steps/s (Qwen3-8B-shaped sweep); HBM GB/s
 UNIT = "seq-steps/s"
 WORKLOAD = "qwen3-8b-ladder"
 NOMINAL_HBM_GBS = 8000.0
+# DRAM bytes per algorithmic byte of a kernel, from one ncu capture of the
+# reduced ladder case (read + written bytes / algorithmic bytes of that launch);
+# traffic grows in proportion to the units a launch processes.  Only kernels
+# whose current build was captured are listed.
+TRAFFIC_PER_ALGORITHMIC_BYTE = {"generated_span_pass": 553.78 / 538.97}
 
 
 def step_schedule(T: int, n: int, offset: int = 0):
     """Decode steps at the midpoints of n equal slices of 1..T."""
     return [1 + ((2 * ((k + offset) % n) + 1) * T) // (2 * n) for k in range(n)]
+
+
+def rank_batch(num_batches: int, base: int, rank: int) -> int:
+    """Weak scaling: rank r of the job runs sweep batch (base + r) mod #batches."""
+    return (base + rank) % num_batches
+
+
+def reduce_timing(ms: float, units: int, dist=None, device=None):
+    """Whole-job timing: the slowest rank's time and the units of all ranks."""
+    if dist is None or not dist.is_initialized() or dist.get_world_size() == 1:
+        return ms, units
+    import torch
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    u = torch.tensor([units], dtype=torch.float64, device=device)
+    dist.all_reduce(u)
+    return float(t.item()), int(u.item())
 
 
 def read_peaks():
@@ -283,7 +305,7 @@ def gpu_arm(args):
     torch.cuda.set_device(local)
     B.build()
     wl = W.get(args.workload)
-    batch = (args.batch + rank) % wl.num_batches()   # weak scaling: one sweep batch per GPU
+    batch = rank_batch(wl.num_batches(), args.batch, rank)
     sb = SweepBatch(wl, batch)
     N = wl.num_layers
     steps = step_schedule(wl.max_steps, args.steps)
@@ -334,13 +356,7 @@ def gpu_arm(args):
     S.splice_check_device_error(sb.desc)
 
     units = sb.B * len(steps)
-    if world > 1:
-        tt = torch.tensor([ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
-        uu = torch.tensor([units], device=dev, dtype=torch.float64)
-        dist.all_reduce(uu)
-        units = int(uu.item())
+    ms, units = reduce_timing(ms, units, dist if world > 1 else None, dev)
     value = units / (ms / 1000.0)
 
     # ---- algorithmic bytes of the timed steps ----
@@ -385,12 +401,14 @@ def gpu_arm(args):
                        "decode_steps_t": steps, "l2": "inputs larger than L2 (every step streams >10 GB); no flush",
                        "parallelism": f"{world} GPU(s), one sweep batch each, no collective"},
             "hbm": {"algorithmic_GB_per_step": round(total_bytes / len(steps) / 1e9, 3),
-                    "achieved_GBps": round(total_bytes / (ms / 1000.0) / 1e9 / max(world, 1) * max(world, 1), 1),
+                    "achieved_GBps": round(total_bytes / (ms / 1000.0) / 1e9, 1),
                     "frac_of_measured": round(total_bytes / (ms / 1000.0) / 1e9 / peak, 4),
                     "frac_of_8TBps": round(total_bytes / (ms / 1000.0) / 1e9 / NOMINAL_HBM_GBS, 4)},
             "roofline": {"kernel": dom, "bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
                          "unit": "GB/s", "frac": round(achieved / peak, 4), "peak_source": peak_kind,
-                         "traffic": None, "bytes_per_launch": per_kind[dom] // max(n_l, 1),
+                         "traffic": (round(TRAFFIC_PER_ALGORITHMIC_BYTE[dom] * per_kind[dom] / max(n_l, 1))
+                                     if dom in TRAFFIC_PER_ALGORITHMIC_BYTE else None),
+                         "bytes_per_launch": per_kind[dom] // max(n_l, 1),
                          "ms_per_launch": ms_l / max(n_l, 1)},
             "kernels": kernels,
             "e2e": e2e, "gpu_launches": gpu_launches, "clocks": clk.summary(), "cpu_baseline": cpu,

@@ -263,6 +263,13 @@ splice_status splice_profile_enable(splice_desc* desc, int enable);
 splice_status splice_profile_read(splice_desc* desc, long long* launches, double* total_ms);
 const char* splice_kernel_kind_name(int kind);
 
+/* Test of the failure path: launches one thread whose mbarrier wait can never
+ * complete and gives up after limit_us microseconds (1 .. 1000000), recording
+ * an error bit in the descriptor's error word exactly as a streaming kernel's
+ * bounded wait would; splice_check_device_error then returns SPLICE_EDEVICE.
+ * Nothing faults or hangs. */
+splice_status splice_debug_wait_timeout(splice_desc* desc, unsigned limit_us, void* stream);
+
 /* Static description of a status code. */
 const char* splice_status_str(splice_status status);
 

@@ -506,6 +506,17 @@ splice_status splice_check_device_error(splice_desc* d) {
     return SPLICE_OK;
 }
 
+splice_status splice_debug_wait_timeout(splice_desc* d, unsigned limit_us, void* stream) {
+    if (!d) return fail(SPLICE_EINVAL, "NULL descriptor");
+    if (!d->on_device) return fail(SPLICE_ESTATE, "host-only descriptor");
+    if (limit_us == 0 || limit_us > 1000000u) return fail(SPLICE_EINVAL, "limit_us %u not in [1, 1000000]", limit_us);
+    DeviceGuard g(d->device);
+    if (g.err != cudaSuccess) return cuda_fail(g.err, "cudaSetDevice");
+    cudaError_t e = cudaError_t(splice::launch_wait_timeout(d->d_err, 1000ull * limit_us, stream));
+    if (e != cudaSuccess) return cuda_fail(e, "wait-timeout launch");
+    return SPLICE_OK;
+}
+
 long long splice_kernel_launches(const splice_desc* d) { return d ? d->launches : -1; }
 
 splice_status splice_profile_enable(splice_desc* d, int enable) {

@@ -98,6 +98,9 @@ int launch_generated_span(const AttnParams& p, void* stream);
 int generated_span_resident_warps(int d);
 int launch_merge(const AttnParams& p, void* stream);
 
+// One-thread kernel whose mbarrier wait runs out after limit_ns.
+int launch_wait_timeout(unsigned* err, unsigned long long limit_ns, void* stream);
+
 // Tensor-core prompt-span pass.  A tensor map is a 128-byte CUtensorMap.
 int make_kv_tensor_map(void* out_map, const void* base, long rows, int d, int box_rows);
 int prefix_tc_box_rows(int d);

@@ -59,6 +59,7 @@ SIGNATURES = {
     "splice_plan_stats": (_c_int, [_vp, _c_int, _c_int, ctypes.POINTER(_c_int), ctypes.POINTER(_c_int),
                                    ctypes.POINTER(_c_int), ctypes.POINTER(_c_int)]),
     "splice_check_device_error": (_c_int, [_vp]),
+    "splice_debug_wait_timeout": (_c_int, [_vp, ctypes.c_uint, _vp]),
     "splice_kernel_launches": (ctypes.c_longlong, [_vp]),
     "splice_profile_enable": (_c_int, [_vp, _c_int]),
     "splice_profile_read": (_c_int, [_vp, ctypes.POINTER(ctypes.c_longlong), ctypes.POINTER(ctypes.c_double)]),
@@ -210,6 +211,10 @@ def splice_plan_stats(desc: Desc, layer, step) -> dict:
     _check(lib().splice_plan_stats(desc.handle, layer, step, ctypes.byref(g), ctypes.byref(t),
                                    ctypes.byref(p), ctypes.byref(s)), "splice_plan_stats")
     return {"num_groups": g.value, "num_tiles": t.value, "prompt_visible": p.value, "suffix_visible": s.value}
+
+
+def splice_debug_wait_timeout(desc: Desc, limit_us: int, stream=None):
+    _check(lib().splice_debug_wait_timeout(desc.handle, limit_us, _stream(stream)), "splice_debug_wait_timeout")
 
 
 def splice_check_device_error(desc: Desc):

@@ -162,3 +162,19 @@ def test_argument_errors_on_device_descriptor():
         S.suffix_kv_append(a.desc, 0, 0, a.k_new, a.v_new, a.k_suffix, a.v_suffix)
     assert e.value.status == S.EINVAL
     S.splice_check_device_error(a.desc)
+
+
+def test_bounded_wait_reports_instead_of_hanging():
+    """A wait that can never complete gives up after its limit and the host
+    reads SPLICE_EDEVICE; the context stays usable and the record clears."""
+    wl = small_wl()
+    a = SweepBatch(wl, seqs=wl.sequences())
+    S.splice_check_device_error(a.desc)
+    S.splice_debug_wait_timeout(a.desc, 1000)          # 1 ms
+    with pytest.raises(S.SpliceError) as e:
+        S.splice_check_device_error(a.desc)
+    assert e.value.status == S.EDEVICE
+    S.splice_check_device_error(a.desc)                # cleared
+    out = a.run(1, 5).clone()                           # the GPU still works
+    assert torch.isfinite(out).all()
+    S.splice_check_device_error(a.desc)
