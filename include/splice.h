@@ -32,7 +32,10 @@
  *     call.  splice_last_error() gives a one-line reason for the last
  *     failure on the calling thread.
  *   - A descriptor is not thread-safe: do not use one descriptor from two
- *     host threads at once.
+ *     host threads at once.  Launches that use one descriptor must not
+ *     overlap on the GPU either (issue them on one stream, or order them
+ *     with events): its device tables hold the error word and the work
+ *     counter that the prompt-span pass hands out work with.
  */
 #ifndef SPLICE_H
 #define SPLICE_H

@@ -37,6 +37,7 @@ struct splice_desc {
     int32_t* d_group_src = nullptr;
     int32_t* d_group_seqs = nullptr;
     unsigned* d_err = nullptr;
+    unsigned* d_sched = nullptr;   // [2] prompt-span work counter, finished-CTA count (zero between launches)
     // Measurement: launch counter and optional per-launch event timing.
     long long launches = 0;
     bool profiling = false;
@@ -252,6 +253,7 @@ splice_status splice_desc_create(const splice_model_shape* sh, int P, int Tp, in
         seq_slot[s] = d->seqs[s].donor_slot;
     }
     const unsigned zero = 0;
+    const unsigned sched_zero[2] = {0, 0};
     Part parts[] = {
         {pl.src.data(), pl.src.size(), 0},
         {seq_prompt.data(), seq_prompt.size() * 4, 0},
@@ -262,6 +264,7 @@ splice_status splice_desc_create(const splice_model_shape* sh, int P, int Tp, in
         {pl.group_src.data(), pl.group_src.size() * 4, 0},
         {pl.group_seqs.data(), pl.group_seqs.size() * 4, 0},
         {&zero, sizeof zero, 0},
+        {sched_zero, sizeof sched_zero, 0},
     };
     size_t total = 0;
     for (Part& p : parts) {
@@ -300,6 +303,7 @@ splice_status splice_desc_create(const splice_model_shape* sh, int P, int Tp, in
     d->d_group_src = reinterpret_cast<int32_t*>(b + parts[6].off);
     d->d_group_seqs = reinterpret_cast<int32_t*>(b + parts[7].off);
     d->d_err = reinterpret_cast<unsigned*>(b + parts[8].off);
+    d->d_sched = reinterpret_cast<unsigned*>(b + parts[9].off);
     d->on_device = true;
     *out = d;
     return SPLICE_OK;
@@ -397,6 +401,7 @@ splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const spl
     p.group_src = d->d_group_src;
     p.group_seqs = d->d_group_seqs;
     p.err = d->d_err;
+    p.sched = d->d_sched;
     p.B = d->B;
     p.N = sh.num_layers;
     p.Hq = sh.num_q_heads;

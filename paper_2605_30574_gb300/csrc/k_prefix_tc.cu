@@ -4,22 +4,29 @@
 // step) -- a group of the descriptor's table -- shares that span's K/V.  For
 // one kv head h, the G query rows of every sequence of the group are stacked
 // into 128-row tiles, so Q K^T and P V over the span are dense contractions
-// (M = 128 stacked rows).  A work item is one (row tile, kv head, key split);
-// each CTA walks a fixed stream of items:
+// (M = 128 stacked rows).  A work item is one (row tile, kv head, key
+// split).  Items are handed out at run time: each CTA's producer claims the
+// next item from a launch-wide counter and posts it to the CTA's other roles
+// through a small ring in smem, so CTAs that draw short items take more.
 //
-//   warp 0        TMA producer: K and V blocks of the item's span -> a
-//                 two-stage smem ring, running ahead across item boundaries
-//   warp 1        MMA issuer (one lane): S = Q K^T into TMEM (two buffers);
-//                 O += P V with P read from TMEM; O double-buffered in TMEM
-//                 when it fits; owns the TMEM allocation
-//   warp 2        Q gather: the tile's query rows -> smem (double-buffered),
+//   warp 0        TMA producer: claims items; K and V blocks of the item's
+//                 span -> a two-stage smem ring, running ahead across items
+//   warp 1        Q K^T issuer (one elected lane): S of the next key block
+//                 into a free TMEM slot (NSLOT slots); owns the TMEM
+//                 allocation
+//   warp 2        Q gather: the tile's query rows -> smem with cp.async,
 //                 one item ahead
 //   warps 3..10   softmax, two warpgroups: each thread owns one row and one
-//                 half of every key block; the halves trade block maxima
+//                 half of every block's keys; the halves trade block maxima
 //                 through smem, share one lazily moved reference max, write
-//                 P (bf16) over their own half of S in TMEM, rescale their
-//                 half of O when the reference moves, and at the item's end
-//                 write the row's partial state (m, l, o) to the workspace.
+//                 P (bf16) over their own half of the slot in TMEM, rescale
+//                 their half of O when the reference moves, and at the item's
+//                 end write the row's partial state (m, l, o) to the
+//                 workspace.  Warps whose 32 rows are all past the tile's end
+//                 skip the arithmetic but keep every barrier.
+//   warp 11       P V issuer (one elected lane): O += P V with P read from
+//                 TMEM as soon as the softmax has written it -- a separate
+//                 issuer, so P V never queues behind the next Q K^T
 //
 // The merge kernel combines these partials with those of the generated span
 // (and the ZERO closed form).  Every wait is bounded: a wait that runs out
@@ -38,15 +45,18 @@
 namespace splice {
 namespace {
 
-constexpr int kRows = 128;          // MMA M
-constexpr int kWarps = 11;
+constexpr int kRows = 128;          // MMA M, rows of one tile
+constexpr int kWarps = 12;          // producer, Q K^T issuer, Q gather, 8 softmax, P V issuer
+constexpr int kPvWarp = 11;
 constexpr int kThreads = kWarps * 32;
-constexpr int kSoftmaxThreads = 256;
 constexpr uint32_t kTmemCols = 512;
 constexpr float kTau = 8.0f;        // lazy rescale threshold, log2 units
 
 constexpr unsigned kErrWaitProducer = 0x1, kErrWaitMma = 0x2, kErrWaitSoftmax = 0x4, kErrWaitDrain = 0x8,
-                   kErrWaitQ = 0x20;
+                   kErrWaitQ = 0x20, kErrWaitItem = 0x40;
+// Work items reach the CTA's roles through a ring of item numbers in smem.
+constexpr int kItemRing = 8;
+constexpr int kItemTakers = 11;     // Q K^T warp, P V warp, Q gather warp, 8 softmax warps
 
 __device__ __forceinline__ float ex2(float x) {
     float y;
@@ -75,26 +85,52 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&v)[16
 
 template <int D>
 struct Cfg {
-    static constexpr int BN = D == 256 ? 64 : 128;          // keys per block
-    static constexpr int HALF = BN / 2;                     // keys per softmax thread per block
-    static constexpr int STAGES = 2;
-    static constexpr int KB = D / 64;                         // 64-wide K blocks of Q / K tile
-    static constexpr uint32_t Q_BYTES = kRows * D * 2;
-    static constexpr uint32_t KV_BYTES = BN * D * 2;          // one K (or V) block
-    static constexpr int NO = (2 * BN + 2 * D <= int(kTmemCols)) ? 2 : 1;   // O buffers in TMEM
-    static constexpr int NQ = (2 * Q_BYTES + 4 * KV_BYTES <= 200u * 1024u) ? 2 : 1;   // Q buffers in smem
-    static constexpr uint32_t OFF_Q = 0;                      // [NQ] Q buffers
+    static constexpr int BN = D == 256 ? 64 : 128;          // keys per K/V block
+    static constexpr int KPT = BN / 2;                      // keys per softmax thread per block
+    static constexpr int OCH = D / 2;                       // O columns per softmax thread
+    static constexpr int KB = D / 64;                       // 64-wide column blocks of Q / K / V
+    static constexpr uint32_t KV_BYTES = BN * D * 2;        // one K (or V) block
+    static constexpr int STAGES = int((64u * 1024u) / KV_BYTES);   // 64 KB of K and 64 KB of V in flight
+    static constexpr uint32_t Q_BYTES = kRows * D * 2;      // Q of one tile
+    static constexpr int NQ = (2 * Q_BYTES + 2 * STAGES * KV_BYTES <= 200u * 1024u) ? 2 : 1;   // Q buffers
+    // TMEM columns: NSLOT slots of BN columns for S (each softmax thread's
+    // P over the first columns of its half of the slot), then O.
+    static constexpr int NSLOT = (int(kTmemCols) - D) / BN > 4 ? 4 : (int(kTmemCols) - D) / BN;
+    static constexpr uint32_t COL_O = NSLOT * BN;
+    static constexpr uint32_t OFF_Q = 0;                    // [NQ] Q buffers
     static constexpr uint32_t OFF_K = OFF_Q + NQ * Q_BYTES;
     static constexpr uint32_t OFF_V = OFF_K + STAGES * KV_BYTES;
-    static constexpr uint32_t OFF_X = OFF_V + STAGES * KV_BYTES;   // [2 parity][2 wg][128] max exchange
-    static constexpr uint32_t OFF_LX = OFF_X + 2 * 2 * kRows * 4;    // [128] l exchange
-    static constexpr uint32_t OFF_BAR = OFF_LX + kRows * 4;
-    static constexpr uint32_t SMEM = OFF_BAR + 256 + 1024;    // + barriers, + alignment slack
-    // TMEM columns: S buffers at 0 and BN (P overwrites each half's first
-    // quarter), O buffers after them.
-    static constexpr uint32_t COL_S = 0, COL_O = 2 * BN;
-    static_assert(2 * BN + NO * D <= int(kTmemCols), "TMEM budget");
+    // exchange: [2 parity][2 half][128] block maxima, [2 parity][2 half][128] row sums
+    static constexpr uint32_t OFF_X = OFF_V + STAGES * KV_BYTES;
+    static constexpr uint32_t X_BYTES = 2 * (2 * 2 * kRows) * 4;
+    static constexpr uint32_t OFF_BAR = OFF_X + X_BYTES;
+    static constexpr uint32_t SMEM = OFF_BAR + 1024 + 1024;   // + barriers, + alignment slack
+    static_assert(NSLOT >= 2 && COL_O + D <= kTmemCols, "TMEM budget");
     static_assert(SMEM <= 227 * 1024, "shared memory budget");
+    static_assert(KPT % 32 == 0 && OCH % 32 == 0 && STAGES >= 2, "TMEM access granularity, ring depth");
+};
+
+// Barrier indices (8 bytes each from OFF_BAR).
+template <int STAGES, int NSLOT>
+struct Bars {
+    static constexpr int KFULL = 0;                       // [STAGES]
+    static constexpr int KEMPTY = STAGES;                 // [STAGES]
+    static constexpr int VFULL = 2 * STAGES;              // [STAGES]
+    static constexpr int VEMPTY = 3 * STAGES;             // [STAGES]
+    static constexpr int SFULL = 4 * STAGES;              // [NSLOT] S computed
+    static constexpr int SFREE = SFULL + NSLOT;           // [NSLOT] P of the slot consumed by P V
+    static constexpr int PFULL = SFREE + NSLOT;           // [NSLOT] P written (and O rescaled)
+    static constexpr int QFULL = PFULL + NSLOT;           // [2]
+    static constexpr int QEMPTY = QFULL + 2;              // [2]
+    static constexpr int ODONE = QEMPTY + 2;
+    static constexpr int OFREE = ODONE + 1;
+    static constexpr int DRAIN = OFREE + 1;               // [issuer]
+    static constexpr int XCH = DRAIN + 2;                 // [2] block-maximum exchange
+    static constexpr int LXCH = XCH + 2;                  // row-sum exchange at an item's end
+    static constexpr int IFULL = LXCH + 1;                // [kItemRing] item number posted
+    static constexpr int IEMPTY = IFULL + kItemRing;      // [kItemRing] item number taken by every role
+    static constexpr int COUNT = IEMPTY + kItemRing;
+    static_assert(COUNT * 8 + 16 + 4 * kItemRing <= 1024, "barrier area");
 };
 
 struct TcParams {
@@ -104,28 +140,11 @@ struct TcParams {
     int n_items;
 };
 
-enum : int {
-    B_KFULL = 0,    // [2]
-    B_KEMPTY = 2,   // [2]
-    B_VFULL = 4,    // [2]
-    B_VEMPTY = 6,   // [2]
-    B_SFULL = 8,    // [2] S block computed
-    B_SFREE = 10,   // [2] P of the block consumed by P V (S buffer reusable, O updated)
-    B_PFULL = 12,   // [2] P written (and O rescaled) by the softmax threads
-    B_QFULL = 14,   // [2]
-    B_QEMPTY = 16,  // [2]
-    B_ODONE = 18,   // [2]
-    B_OFREE = 20,   // [2]
-    B_DRAIN = 22,
-    B_XCH = 23,     // [2] block-maximum exchange between the two softmax halves
-    B_LXCH = 25,    // row-sum exchange at an item's end
-    B_COUNT = 26
-};
-
-// Decode work item -> tile, kv head, split (consecutive items = consecutive
-// tiles of one (head, split), so a group's tiles read its span together).
+// Work item -> tile, kv head, split (consecutive items = consecutive tiles
+// of one (head, split), so a group's tiles read its span at about the same
+// time and share it in L2).
 struct ItemInfo {
-    int tile, h, split, grp, first, nseq, k0, k1, nblk;
+    int h, split, first, nseq, k0, k1, nblk;
     long span_row;      // first row of the span in the store's 2D view
     bool donor;
 };
@@ -133,16 +152,15 @@ struct ItemInfo {
 template <int D>
 __device__ __forceinline__ ItemInfo item_info(const AttnParams& P, const TcParams& tp, int item) {
     ItemInfo it;
-    it.tile = item % P.n_tiles;
+    const int tile = item % P.n_tiles;
     const int hs = item / P.n_tiles;
     it.split = hs % tp.nsplit;
     it.h = hs / tp.nsplit;
-    const int4 tl = reinterpret_cast<const int4*>(P.tiles)[it.tile];
-    it.grp = tl.x;
+    const int4 tl = reinterpret_cast<const int4*>(P.tiles)[tile];
     it.first = tl.y;
     it.nseq = tl.z;
-    const int prompt = P.group_prompt[it.grp];
-    const int code = P.group_src[it.grp];
+    const int prompt = P.group_prompt[tl.x];
+    const int code = P.group_src[tl.x];
     it.donor = code != int(SPLICE_SRC_CLEAN);
     long span;
     if (!it.donor) {
@@ -164,34 +182,44 @@ __global__ void __launch_bounds__(kThreads, 1)
                      const __grid_constant__ CUtensorMap tm_kd, const __grid_constant__ CUtensorMap tm_vd,
                      const TcParams tp) {
     using C = Cfg<D>;
+    using Bb = Bars<C::STAGES, C::NSLOT>;
+    constexpr int NSLOT = C::NSLOT;
     const AttnParams& P = tp.a;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const uint32_t sbase = tc::smem_u32(smem);
     const uint32_t bar0 = sbase + C::OFF_BAR;
     auto bar = [&](int i) { return bar0 + 8u * uint32_t(i); };
-    volatile int* s_abort = reinterpret_cast<volatile int*>(smem + C::OFF_BAR + 8 * B_COUNT);
-    uint32_t* s_tmem = reinterpret_cast<uint32_t*>(smem + C::OFF_BAR + 8 * B_COUNT + 8);
+    volatile int* s_abort = reinterpret_cast<volatile int*>(smem + C::OFF_BAR + 8 * Bb::COUNT);
+    uint32_t* s_tmem = reinterpret_cast<uint32_t*>(smem + C::OFF_BAR + 8 * Bb::COUNT + 8);
+    volatile int* s_items = reinterpret_cast<volatile int*>(smem + C::OFF_BAR + 8 * Bb::COUNT + 16);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < 2; ++i) {
-            tc::mbar_init(bar(B_KFULL + i), 1);
-            tc::mbar_init(bar(B_KEMPTY + i), 1);
-            tc::mbar_init(bar(B_VFULL + i), 1);
-            tc::mbar_init(bar(B_VEMPTY + i), 1);
-            tc::mbar_init(bar(B_SFULL + i), 1);
-            tc::mbar_init(bar(B_SFREE + i), 1);
-            tc::mbar_init(bar(B_PFULL + i), kSoftmaxThreads);
-            tc::mbar_init(bar(B_QFULL + i), 32);
-            tc::mbar_init(bar(B_QEMPTY + i), 1);
-            tc::mbar_init(bar(B_ODONE + i), 1);
-            tc::mbar_init(bar(B_OFREE + i), kSoftmaxThreads);
+        for (int i = 0; i < C::STAGES; ++i) {
+            tc::mbar_init(bar(Bb::KFULL + i), 1);
+            tc::mbar_init(bar(Bb::KEMPTY + i), 1);
+            tc::mbar_init(bar(Bb::VFULL + i), 1);
+            tc::mbar_init(bar(Bb::VEMPTY + i), 1);
         }
-        tc::mbar_init(bar(B_DRAIN), 1);
-        tc::mbar_init(bar(B_XCH), kSoftmaxThreads);
-        tc::mbar_init(bar(B_XCH + 1), kSoftmaxThreads);
-        tc::mbar_init(bar(B_LXCH), kSoftmaxThreads);
+        for (int i = 0; i < NSLOT; ++i) {
+            tc::mbar_init(bar(Bb::SFULL + i), 1);
+            tc::mbar_init(bar(Bb::SFREE + i), 1);
+            tc::mbar_init(bar(Bb::PFULL + i), 256);
+        }
+        for (int i = 0; i < 2; ++i) {
+            tc::mbar_init(bar(Bb::QFULL + i), 32);
+            tc::mbar_init(bar(Bb::QEMPTY + i), 1);
+            tc::mbar_init(bar(Bb::XCH + i), 256);
+            tc::mbar_init(bar(Bb::DRAIN + i), 1);
+        }
+        tc::mbar_init(bar(Bb::ODONE), 1);
+        tc::mbar_init(bar(Bb::OFREE), 256);
+        tc::mbar_init(bar(Bb::LXCH), 256);
+        for (int i = 0; i < kItemRing; ++i) {
+            tc::mbar_init(bar(Bb::IFULL + i), 1);
+            tc::mbar_init(bar(Bb::IEMPTY + i), kItemTakers);
+        }
         *s_abort = 0;
         tc::fence_mbar_init();
     }
@@ -209,13 +237,40 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc::tc_fence_after();
     const uint32_t tmem = *s_tmem;
+    // Item k of the CTA's stream, for a whole warp: -1 after the last item,
+    // -2 when the wait gave up.
+    auto take_item = [&](int k) -> int {
+        const int r = k % kItemRing;
+        if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::IFULL + r), uint32_t(k / kItemRing) & 1u, s_abort, P.err,
+                                                   kErrWaitItem)))
+            return -2;
+        const int item = s_items[r];
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(bar(Bb::IEMPTY + r));
+        return item;
+    };
+    // Key block number g of the CTA's stream (counted over all its items)
+    // uses S slot g mod NSLOT, for the (g / NSLOT)-th time.
+    auto col_s = [](int g) { return uint32_t((g % NSLOT) * C::BN); };
+    auto use_of = [](int g) { return uint32_t(g / NSLOT) & 1u; };
 
     if (warp == 0) {
         // ------------------------------------------------ TMA producer
         if (lane == 0) {
             int jg = 0;          // global block counter of this CTA
             int issued_k = 0, issued_v = 0;
-            for (int item = blockIdx.x; item < tp.n_items && !*s_abort; item += gridDim.x) {
+            int nxt = int(atomicAdd(P.sched, 1u));
+            for (int k = 0; !*s_abort; ++k) {
+                // post the next item to the other roles
+                const int r = k % kItemRing;
+                if (!tc::mbar_wait(bar(Bb::IEMPTY + r), (uint32_t(k / kItemRing) & 1u) ^ 1u, s_abort, P.err,
+                                   kErrWaitProducer))
+                    break;
+                const int item = nxt < tp.n_items ? nxt : -1;
+                s_items[r] = item;
+                tc::mbar_arrive(bar(Bb::IFULL + r));
+                if (item < 0) break;
+                nxt = int(atomicAdd(P.sched, 1u));   // claimed now, needed after this item's copies
                 const ItemInfo it = item_info<D>(P, tp, item);
                 const CUtensorMap* tmk = it.donor ? &tm_kd : &tm_kc;
                 const CUtensorMap* tmv = it.donor ? &tm_vd : &tm_vc;
@@ -223,158 +278,173 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int stg = jg % C::STAGES;
                     const uint32_t use = uint32_t(jg / C::STAGES);
                     const int y = int(it.span_row + it.k0 + j * C::BN);
-                    if (!tc::mbar_wait(bar(B_KEMPTY + stg), (use & 1u) ^ 1u, s_abort, P.err, kErrWaitProducer)) break;
-                    tc::mbar_arrive_expect_tx(bar(B_KFULL + stg), C::KV_BYTES);
+                    if (!tc::mbar_wait(bar(Bb::KEMPTY + stg), (use & 1u) ^ 1u, s_abort, P.err, kErrWaitProducer))
+                        break;
+                    tc::mbar_arrive_expect_tx(bar(Bb::KFULL + stg), C::KV_BYTES);
 #pragma unroll
                     for (int b = 0; b < C::KB; ++b)
                         tc::tma_load_2d(sbase + C::OFF_K + stg * C::KV_BYTES + b * (C::BN * 128), tmk, b * 64, y,
-                                        bar(B_KFULL + stg));
+                                        bar(Bb::KFULL + stg));
                     issued_k = jg + 1;
-                    if (!tc::mbar_wait(bar(B_VEMPTY + stg), (use & 1u) ^ 1u, s_abort, P.err, kErrWaitProducer)) break;
-                    tc::mbar_arrive_expect_tx(bar(B_VFULL + stg), C::KV_BYTES);
+                    if (!tc::mbar_wait(bar(Bb::VEMPTY + stg), (use & 1u) ^ 1u, s_abort, P.err, kErrWaitProducer))
+                        break;
+                    tc::mbar_arrive_expect_tx(bar(Bb::VFULL + stg), C::KV_BYTES);
 #pragma unroll
                     for (int b = 0; b < C::KB; ++b)
                         tc::tma_load_2d(sbase + C::OFF_V + stg * C::KV_BYTES + b * (C::BN * 128), tmv, b * 64, y,
-                                        bar(B_VFULL + stg));
+                                        bar(Bb::VFULL + stg));
                     issued_v = jg + 1;
                 }
             }
             // Drain: every issued copy must land before the CTA may exit.
             for (int j = max(0, issued_k - C::STAGES); j < issued_k; ++j) {
                 volatile int no_abort = 0;
-                tc::mbar_wait(bar(B_KFULL + j % C::STAGES), uint32_t(j / C::STAGES) & 1u, &no_abort, P.err,
+                tc::mbar_wait(bar(Bb::KFULL + j % C::STAGES), uint32_t(j / C::STAGES) & 1u, &no_abort, P.err,
                               kErrWaitDrain);
             }
             for (int j = max(0, issued_v - C::STAGES); j < issued_v; ++j) {
                 volatile int no_abort = 0;
-                tc::mbar_wait(bar(B_VFULL + j % C::STAGES), uint32_t(j / C::STAGES) & 1u, &no_abort, P.err,
+                tc::mbar_wait(bar(Bb::VFULL + j % C::STAGES), uint32_t(j / C::STAGES) & 1u, &no_abort, P.err,
                               kErrWaitDrain);
             }
         }
     } else if (warp == 1) {
-        // ------------------------------------------------ MMA issuer
-        if (lane == 0) {
-            constexpr uint32_t idesc_qk = tc::idesc_bf16_f32(kRows, C::BN, false);
-            constexpr uint32_t idesc_pv = tc::idesc_bf16_f32(kRows, D, true);
-            bool ok = true, committed = false;
-            int jg = 0, n_item = 0;
-            for (int item = blockIdx.x; ok && item < tp.n_items; item += gridDim.x, ++n_item) {
-                const ItemInfo it = item_info<D>(P, tp, item);
-                const int qb = C::NQ == 2 ? (n_item & 1) : 0;
-                const uint32_t quse = uint32_t(C::NQ == 2 ? n_item >> 1 : n_item);
-                const int ob = C::NO == 2 ? (n_item & 1) : 0;
-                const uint32_t ouse = uint32_t(C::NO == 2 ? n_item >> 1 : n_item);
-                const uint32_t q_addr = sbase + C::OFF_Q + qb * C::Q_BYTES;
-                const uint32_t o_col = tmem + C::COL_O + ob * D;
-                if (!tc::mbar_wait(bar(B_QFULL + qb), quse & 1u, s_abort, P.err, kErrWaitMma)) {
+        // ------------------------------------------------ Q K^T issuer
+        // The whole warp runs the loop; one elected lane issues the MMAs and
+        // their commits.
+        const bool leader = tc::elect_one();
+        constexpr uint32_t idesc_qk = tc::idesc_bf16_f32(kRows, C::BN, false);
+        bool ok = true, committed = false;
+        int jg = 0;
+        for (int k = 0;; ++k) {
+            const int item = take_item(k);
+            if (item < 0) {
+                ok = item == -1;
+                break;
+            }
+            const ItemInfo it = item_info<D>(P, tp, item);
+            const int qb = C::NQ == 2 ? (k & 1) : 0;
+            const uint32_t quse = uint32_t(C::NQ == 2 ? k >> 1 : k);
+            const uint32_t q_addr = sbase + C::OFF_Q + qb * C::Q_BYTES;
+            if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::QFULL + qb), quse & 1u, s_abort, P.err, kErrWaitMma))) {
+                ok = false;
+                break;
+            }
+            for (int j = 0; j < it.nblk; ++j, ++jg) {
+                const int stg = jg % C::STAGES;
+                const int slot = jg % NSLOT;
+                // the K block is loaded, and the slot's previous P V is done
+                if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::KFULL + stg), uint32_t(jg / C::STAGES) & 1u, s_abort,
+                                                           P.err, kErrWaitMma)) ||
+                    !__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::SFREE + slot), use_of(jg) ^ 1u, s_abort, P.err,
+                                                           kErrWaitMma))) {
                     ok = false;
                     break;
                 }
-                auto pv = [&](int jgp, int jl) -> bool {
-                    const int stg = jgp % C::STAGES;
-                    const int sb = jgp & 1;
-                    if (!tc::mbar_wait(bar(B_PFULL + sb), uint32_t(jgp >> 1) & 1u, s_abort, P.err, kErrWaitMma))
-                        return false;
-                    if (!tc::mbar_wait(bar(B_VFULL + stg), uint32_t(jgp / C::STAGES) & 1u, s_abort, P.err,
-                                       kErrWaitMma))
-                        return false;
-                    if (jl == 0 &&
-                        !tc::mbar_wait(bar(B_OFREE + ob), (ouse & 1u) ^ 1u, s_abort, P.err, kErrWaitMma))
-                        return false;
-                    tc::tc_fence_after();
-                    const uint32_t v_addr = sbase + C::OFF_V + stg * C::KV_BYTES;
-                    const uint32_t p_col = tmem + C::COL_S + sb * C::BN;
-#pragma unroll
-                    for (int kk = 0; kk < C::BN / 16; ++kk) {
-                        // 16 keys of P: two bf16 per TMEM column; the first
-                        // half's P sits at the start of its S half, the second
-                        // half's at the start of the other S half.
-                        const int half = kk / (C::HALF / 16);
-                        const int kin = kk % (C::HALF / 16);
-                        const uint32_t a = p_col + half * C::HALF + kin * 8;
-                        const uint64_t b = tc::sw128_desc(v_addr + kk * 16 * 128, C::BN * 128, 1024);
-                        mma_f16_ts(o_col, a, b, idesc_pv, (jl > 0 || kk > 0) ? 1u : 0u);
-                    }
-                    tc::mma_commit(bar(B_SFREE + sb));
-                    tc::mma_commit(bar(B_VEMPTY + stg));
-                    committed = true;
-                    return true;
-                };
-                for (int j = 0; j < it.nblk; ++j, ++jg) {
-                    const int stg = jg % C::STAGES;
-                    const int sb = jg & 1;
-                    if (!tc::mbar_wait(bar(B_KFULL + stg), uint32_t(jg / C::STAGES) & 1u, s_abort, P.err, kErrWaitMma) ||
-                        !tc::mbar_wait(bar(B_SFREE + sb), (uint32_t(jg >> 1) & 1u) ^ 1u, s_abort, P.err, kErrWaitMma)) {
-                        ok = false;
-                        break;
-                    }
-                    tc::tc_fence_after();
-                    const uint32_t k_addr = sbase + C::OFF_K + stg * C::KV_BYTES;
+                tc::tc_fence_after();
+                const uint32_t k_addr = sbase + C::OFF_K + stg * C::KV_BYTES;
+                if (leader) {
 #pragma unroll
                     for (int kk = 0; kk < D / 16; ++kk) {
                         const uint64_t a = tc::sw128_desc(q_addr + (kk / 4) * (kRows * 128) + (kk % 4) * 32, 16, 1024);
                         const uint64_t b = tc::sw128_desc(k_addr + (kk / 4) * (C::BN * 128) + (kk % 4) * 32, 16, 1024);
-                        tc::mma_f16_ss(tmem + C::COL_S + sb * C::BN, a, b, idesc_qk, kk > 0 ? 1u : 0u);
+                        tc::mma_f16_ss(tmem + col_s(jg), a, b, idesc_qk, kk > 0 ? 1u : 0u);
                     }
-                    tc::mma_commit(bar(B_SFULL + sb));
-                    tc::mma_commit(bar(B_KEMPTY + stg));
-                    if (j == it.nblk - 1) tc::mma_commit(bar(B_QEMPTY + qb));
-                    committed = true;
-                    if (j >= 1 && !pv(jg - 1, j - 1)) {
-                        ok = false;
-                        break;
-                    }
+                    tc::mma_commit(bar(Bb::SFULL + slot));
+                    tc::mma_commit(bar(Bb::KEMPTY + stg));
+                    if (j == it.nblk - 1) tc::mma_commit(bar(Bb::QEMPTY + qb));
                 }
-                if (!ok) break;
-                if (it.nblk > 0) {
-                    if (!pv(jg - 1, it.nblk - 1)) {
-                        ok = false;
-                        break;
-                    }
-                } else {
-                    tc::mma_commit(bar(B_QEMPTY + qb));
+                committed = true;
+            }
+            if (!ok) break;
+            if (it.nblk == 0 && leader) tc::mma_commit(bar(Bb::QEMPTY + qb));
+        }
+        if (!ok && committed && leader) {
+            // Let the MMAs already issued finish before TMEM is freed.
+            tc::mma_commit(bar(Bb::DRAIN));
+            volatile int no_abort = 0;
+            tc::mbar_wait(bar(Bb::DRAIN), 0, &no_abort, P.err, kErrWaitDrain);
+        }
+    } else if (warp == kPvWarp) {
+        // ------------------------------------------------ P V issuer
+        const bool leader = tc::elect_one();
+        constexpr uint32_t idesc_pv = tc::idesc_bf16_f32(kRows, D, true);
+        bool ok = true, committed = false;
+        int jg = 0;
+        for (int k = 0;; ++k) {
+            const int item = take_item(k);
+            if (item < 0) {
+                ok = item == -1;
+                break;
+            }
+            const ItemInfo it = item_info<D>(P, tp, item);
+            for (int j = 0; j < it.nblk; ++j, ++jg) {
+                const int stg = jg % C::STAGES;
+                const int slot = jg % NSLOT;
+                if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::PFULL + slot), use_of(jg), s_abort, P.err,
+                                                           kErrWaitMma)) ||
+                    !__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::VFULL + stg), uint32_t(jg / C::STAGES) & 1u, s_abort,
+                                                           P.err, kErrWaitMma)) ||
+                    (j == 0 && !__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::OFREE), (uint32_t(k) & 1u) ^ 1u, s_abort,
+                                                                      P.err, kErrWaitMma)))) {
+                    ok = false;
+                    break;
                 }
-                tc::mma_commit(bar(B_ODONE + ob));
+                tc::tc_fence_after();
+                const uint32_t v_addr = sbase + C::OFF_V + stg * C::KV_BYTES;
+                const uint32_t p_col = tmem + col_s(jg);
+                if (leader) {
+#pragma unroll
+                    for (int kk = 0; kk < C::BN / 16; ++kk) {
+                        // 16 keys of P: two bf16 per TMEM column; the first
+                        // half's P sits at the start of the slot, the second
+                        // half's at its middle
+                        const uint32_t a = p_col + (kk / (C::KPT / 16)) * C::KPT + (kk % (C::KPT / 16)) * 8;
+                        const uint64_t b = tc::sw128_desc(v_addr + kk * 16 * 128, C::BN * 128, 1024);
+                        mma_f16_ts(tmem + C::COL_O, a, b, idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
+                    }
+                    tc::mma_commit(bar(Bb::SFREE + slot));
+                    tc::mma_commit(bar(Bb::VEMPTY + stg));
+                }
+                committed = true;
             }
-            if (!ok && committed) {
-                // Let the MMAs already issued finish before TMEM is freed.
-                tc::mma_commit(bar(B_DRAIN));
-                volatile int no_abort = 0;
-                tc::mbar_wait(bar(B_DRAIN), 0, &no_abort, P.err, kErrWaitDrain);
-            }
+            if (!ok) break;
+            if (leader) tc::mma_commit(bar(Bb::ODONE));
+        }
+        if (!ok && committed && leader) {
+            tc::mma_commit(bar(Bb::DRAIN + 1));
+            volatile int no_abort = 0;
+            tc::mbar_wait(bar(Bb::DRAIN + 1), 0, &no_abort, P.err, kErrWaitDrain);
         }
     } else if (warp == 2) {
         // ------------------------------------------------ Q gather
-        int n_item = 0;
-        for (int item = blockIdx.x; item < tp.n_items; item += gridDim.x, ++n_item) {
+        // Rows no item fills keep finite values: zero every buffer once.
+        for (uint32_t off = uint32_t(lane) * 16; off < C::NQ * C::Q_BYTES; off += 32 * 16)
+            *reinterpret_cast<uint4*>(smem + C::OFF_Q + off) = make_uint4(0, 0, 0, 0);
+        __syncwarp();
+        for (int k = 0;; ++k) {
+            const int item = take_item(k);
+            if (item < 0) break;
             const ItemInfo it = item_info<D>(P, tp, item);
-            const int qb = C::NQ == 2 ? (n_item & 1) : 0;
-            const uint32_t quse = uint32_t(C::NQ == 2 ? n_item >> 1 : n_item);
-            const bool got = tc::mbar_wait(bar(B_QEMPTY + qb), (quse & 1u) ^ 1u, s_abort, P.err, kErrWaitQ);
-            if (!__all_sync(0xffffffffu, got)) break;
-            uint8_t* q_s = smem + C::OFF_Q + qb * C::Q_BYTES;
+            const int qb = C::NQ == 2 ? (k & 1) : 0;
+            const uint32_t quse = uint32_t(C::NQ == 2 ? k >> 1 : k);
+            if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::QEMPTY + qb), (quse & 1u) ^ 1u, s_abort, P.err, kErrWaitQ)))
+                break;
+            const uint32_t q_s = sbase + C::OFF_Q + qb * C::Q_BYTES;
             const int nrows = it.nseq * P.G;
 #pragma unroll 1
-            for (int rr = 0; rr < kRows / 32; ++rr) {
-                const int row = rr * 32 + lane;
-                uint4 v[D / 8];
-                if (row < nrows) {
-                    const int s = P.group_seqs[it.first + row / P.G];
-                    const int hq = it.h * P.G + row % P.G;
-                    const uint4* src = reinterpret_cast<const uint4*>(P.q + (long(s) * P.Hq + hq) * D);
-#pragma unroll
-                    for (int c = 0; c < D / 8; ++c) v[c] = src[c];
-                } else {
-#pragma unroll
-                    for (int c = 0; c < D / 8; ++c) v[c] = make_uint4(0, 0, 0, 0);
-                }
+            for (int row = lane; row < nrows; row += 32) {
+                const int s = P.group_seqs[it.first + row / P.G];
+                const int hq = it.h * P.G + row % P.G;
+                const uint16_t* src = P.q + (long(s) * P.Hq + hq) * D;
+                const uint32_t dst = q_s + row * 128;
 #pragma unroll
                 for (int c = 0; c < D / 8; ++c)
-                    *reinterpret_cast<uint4*>(q_s + (c / 8) * (kRows * 128) + row * 128 + (((c % 8) ^ (row % 8)) * 16)) =
-                        v[c];
+                    tc::cp_async16(dst + (c / 8) * (kRows * 128) + (((c % 8) ^ (row % 8)) * 16), src + c * 8);
             }
+            tc::cp_async_wait_all();
             tc::fence_proxy_async_smem();
-            tc::mbar_arrive(bar(B_QFULL + qb));
+            tc::mbar_arrive(bar(Bb::QFULL + qb));
         }
     } else {
         // ------------------------------------------------ softmax / epilogue
@@ -382,192 +452,221 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int quarter = warp & 3;                  // TMEM lane quarter this warp may access
         const int row = quarter * 32 + lane;           // == TMEM lane of this thread's row
         const uint32_t lane_base = uint32_t(quarter * 32) << 16;
-        float* xmax = reinterpret_cast<float*>(smem + C::OFF_X);
-        float* xl = reinterpret_cast<float*>(smem + C::OFF_LX);
+        float* xmax = reinterpret_cast<float*>(smem + C::OFF_X);          // [2][2][128]
+        float* xl = xmax + 2 * 2 * kRows;                                 // [2][2][128]
         const float c = P.scale_log2;
+        const float2 c2 = make_float2(c, c);
         bool ok = true;
-        int jg = 0, n_item = 0, n_lx = 0;
-        for (int item = blockIdx.x; ok && item < tp.n_items; item += gridDim.x, ++n_item) {
+        int jg = 0;
+        for (int k = 0;; ++k) {
+            const int item = take_item(k);
+            if (item < 0) {
+                ok = item == -1;
+                break;
+            }
             const ItemInfo it = item_info<D>(P, tp, item);
-            const int ob = C::NO == 2 ? (n_item & 1) : 0;
-            const uint32_t ouse = uint32_t(C::NO == 2 ? n_item >> 1 : n_item);
-            const bool valid = row < it.nseq * P.G;
-            long out_row = 0;
+            const int nrows = it.nseq * P.G;
+            const bool rows = quarter * 32 < nrows;    // warp-uniform
+            const bool valid = row < nrows;
+            int orow = 0;
             if (valid) {
                 const int s = P.group_seqs[it.first + row / P.G];
-                out_row = long(s) * P.Hq + it.h * P.G + row % P.G;
+                orow = s * P.Hq + it.h * P.G + row % P.G;
             }
             float m_run = -INFINITY, l_run = 0.f;
             for (int j = 0; j < it.nblk; ++j, ++jg) {
-                const int sb = jg & 1;
+                const int slot = jg % NSLOT;
                 // waits are made warp-uniform: tcgen05.ld/st are warp-collective
-                if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(B_SFULL + sb), uint32_t(jg >> 1) & 1u, s_abort, P.err,
+                if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::SFULL + slot), use_of(jg), s_abort, P.err,
                                                            kErrWaitSoftmax))) {
                     ok = false;
                     break;
                 }
-                tc::tc_fence_after();
-                const uint32_t s_col = tmem + lane_base + C::COL_S + sb * C::BN + wg * C::HALF;
-                float s[C::HALF];
+                const uint32_t s_col = tmem + lane_base + col_s(jg) + wg * C::KPT;
+                const int kbase = it.k0 + j * C::BN + wg * C::KPT;
+                const bool tail = kbase + C::KPT > it.k1;
+                float s[C::KPT];
+                float e0 = 0.f;
+                if (rows) {
+                    tc::tc_fence_after();
 #pragma unroll
-                for (int q = 0; q < C::HALF / 32; ++q) {
-                    float v[32];
-                    tc::tmem_ld32(s_col + q * 32, v);
+                    for (int q = 0; q < C::KPT / 32; ++q) {
+                        float v[32];
+                        tc::tmem_ld32(s_col + q * 32, v);
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) s[q * 32 + i] = v[i];
-                }
-                tc::tmem_wait_ld();
-                // keys past the split end are masked (only the last block)
-                const int kbase = it.k0 + j * C::BN + wg * C::HALF;
-                const bool tail = kbase + C::HALF > it.k1;
-                if (tail) {
-#pragma unroll
-                    for (int i = 0; i < C::HALF; ++i)
-                        if (kbase + i >= it.k1) s[i] = c >= 0.f ? -INFINITY : INFINITY;
-                }
-                // block extreme of the raw logits in this half (max for c >= 0)
-                float e0 = s[0], e1 = s[1], e2 = s[2], e3 = s[3];
-                if (c >= 0.f) {
-#pragma unroll
-                    for (int i = 4; i < C::HALF; i += 4) {
-                        e0 = fmaxf(e0, s[i]);
-                        e1 = fmaxf(e1, s[i + 1]);
-                        e2 = fmaxf(e2, s[i + 2]);
-                        e3 = fmaxf(e3, s[i + 3]);
+                        for (int i = 0; i < 32; ++i) s[q * 32 + i] = v[i];
                     }
-                    e0 = fmaxf(fmaxf(e0, e1), fmaxf(e2, e3));
-                } else {
+                    tc::tmem_wait_ld();
+                    // keys past the split end are masked (only the last block)
+                    if (tail) {
 #pragma unroll
-                    for (int i = 4; i < C::HALF; i += 4) {
-                        e0 = fminf(e0, s[i]);
-                        e1 = fminf(e1, s[i + 1]);
-                        e2 = fminf(e2, s[i + 2]);
-                        e3 = fminf(e3, s[i + 3]);
+                        for (int i = 0; i < C::KPT; ++i)
+                            if (kbase + i >= it.k1) s[i] = c >= 0.f ? -INFINITY : INFINITY;
                     }
-                    e0 = fminf(fminf(e0, e1), fminf(e2, e3));
+                    // extreme of this half's raw logits (max for c >= 0)
+                    float e1 = s[1], e2 = s[2], e3 = s[3];
+                    e0 = s[0];
+                    if (c >= 0.f) {
+#pragma unroll
+                        for (int i = 4; i < C::KPT; i += 4) {
+                            e0 = fmaxf(e0, s[i]);
+                            e1 = fmaxf(e1, s[i + 1]);
+                            e2 = fmaxf(e2, s[i + 2]);
+                            e3 = fmaxf(e3, s[i + 3]);
+                        }
+                        e0 = fmaxf(fmaxf(e0, e1), fmaxf(e2, e3));
+                    } else {
+#pragma unroll
+                        for (int i = 4; i < C::KPT; i += 4) {
+                            e0 = fminf(e0, s[i]);
+                            e1 = fminf(e1, s[i + 1]);
+                            e2 = fminf(e2, s[i + 2]);
+                            e3 = fminf(e3, s[i + 3]);
+                        }
+                        e0 = fminf(fminf(e0, e1), fminf(e2, e3));
+                    }
                 }
+                // the two halves of the block trade their extremes
                 float* xm = xmax + (jg & 1) * (2 * kRows);
                 xm[wg * kRows + row] = e0;
-                tc::mbar_arrive(bar(B_XCH + (jg & 1)));
-                if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(B_XCH + (jg & 1)), uint32_t(jg >> 1) & 1u, s_abort,
+                tc::mbar_arrive(bar(Bb::XCH + (jg & 1)));
+                if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::XCH + (jg & 1)), uint32_t(jg >> 1) & 1u, s_abort,
                                                            P.err, kErrWaitSoftmax))) {
                     ok = false;
                     break;
                 }
-                const float eo = xm[(wg ^ 1) * kRows + row];
-                const float ext = c >= 0.f ? fmaxf(e0, eo) : fminf(e0, eo);
-                const float mc = ext * c;                      // block max in log2 units
-                float alpha = 1.f;
-                bool resc = false;
-                if (mc > m_run + kTau) {
-                    alpha = ex2(m_run - mc);
-                    resc = j > 0;
-                    m_run = mc;
-                }
-                const float nm = -m_run;
-                float lsum = 0.f;
-                uint32_t pk[C::HALF / 2];
-#pragma unroll
-                for (int i = 0; i < C::HALF / 2; ++i) {
-                    float a = ex2(fmaf(s[2 * i], c, nm));
-                    float b = ex2(fmaf(s[2 * i + 1], c, nm));
-                    if (tail) {
-                        a = kbase + 2 * i < it.k1 ? a : 0.f;
-                        b = kbase + 2 * i + 1 < it.k1 ? b : 0.f;
+                if (rows) {
+                    const float eo = xm[(wg ^ 1) * kRows + row];
+                    const float mc = (c >= 0.f ? fmaxf(e0, eo) : fminf(e0, eo)) * c;   // block max, log2 units
+                    float alpha = 1.f;
+                    bool resc = false;
+                    if (mc > m_run + kTau) {
+                        alpha = ex2(m_run - mc);
+                        resc = j > 0;
+                        m_run = mc;
                     }
-                    lsum += a + b;
-                    const __nv_bfloat162 h2 = __floats2bfloat162_rn(a, b);
-                    pk[i] = *reinterpret_cast<const uint32_t*>(&h2);
-                }
-                if (__any_sync(0xffffffffu, resc)) {
-                    // O must hold P V of every earlier block of this item
-                    if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(B_SFREE + ((jg - 1) & 1)),
-                                                               uint32_t((jg - 1) >> 1) & 1u, s_abort, P.err,
-                                                               kErrWaitSoftmax))) {
-                        ok = false;
-                        break;
+                    const float2 nm2 = make_float2(-m_run, -m_run);
+                    float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
+                    uint32_t pk[C::KPT / 2];
+#pragma unroll
+                    for (int i = 0; i < C::KPT / 2; ++i) {
+                        const float2 z = __ffma2_rn(make_float2(s[2 * i], s[2 * i + 1]), c2, nm2);
+                        float2 e = make_float2(ex2(z.x), ex2(z.y));
+                        if (tail) {
+                            e.x = kbase + 2 * i < it.k1 ? e.x : 0.f;
+                            e.y = kbase + 2 * i + 1 < it.k1 ? e.y : 0.f;
+                        }
+                        if (i & 1)
+                            acc1 = __fadd2_rn(acc1, e);
+                        else
+                            acc0 = __fadd2_rn(acc0, e);
+                        const __nv_bfloat162 h2 = __floats2bfloat162_rn(e.x, e.y);
+                        pk[i] = *reinterpret_cast<const uint32_t*>(&h2);
                     }
-                    tc::tc_fence_after();
+                    l_run = l_run * alpha + ((acc0.x + acc1.x) + (acc0.y + acc1.y));
+                    // P (bf16 pairs) over the first columns of this half of the slot
 #pragma unroll
-                    for (int q = 0; q < D / 64; ++q) {
-                        float v[32];
-                        const uint32_t ta = tmem + lane_base + C::COL_O + ob * D + wg * (D / 2) + q * 32;
-                        tc::tmem_ld32(ta, v);
-                        tc::tmem_wait_ld();
+                    for (int q = 0; q < C::KPT / 32; ++q) {
+                        uint32_t part[16];
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) v[i] *= resc ? alpha : 1.f;
-                        tc::tmem_st32(ta, v);
+                        for (int i = 0; i < 16; ++i) part[i] = pk[q * 16 + i];
+                        tmem_st16(s_col + q * 16, part);
+                    }
+                    if (__any_sync(0xffffffffu, resc)) {
+                        // O must hold P V of every earlier block of this item
+                        const int jp = jg - 1;
+                        if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::SFREE + jp % NSLOT), use_of(jp), s_abort,
+                                                                   P.err, kErrWaitSoftmax))) {
+                            ok = false;
+                            break;
+                        }
+                        tc::tc_fence_after();
+                        const float2 a2 = make_float2(resc ? alpha : 1.f, resc ? alpha : 1.f);
+#pragma unroll
+                        for (int q = 0; q < C::OCH / 32; ++q) {
+                            float v[32];
+                            const uint32_t ta = tmem + lane_base + C::COL_O + wg * C::OCH + q * 32;
+                            tc::tmem_ld32(ta, v);
+                            tc::tmem_wait_ld();
+#pragma unroll
+                            for (int i = 0; i < 32; i += 2) {
+                                const float2 r = __fmul2_rn(make_float2(v[i], v[i + 1]), a2);
+                                v[i] = r.x;
+                                v[i + 1] = r.y;
+                            }
+                            tc::tmem_st32(ta, v);
+                        }
                     }
                     tc::tmem_wait_st();
                 }
-                l_run = l_run * alpha + lsum;
-                // P (bf16 pairs) over the first quarter of this half's S columns
-                const uint32_t p_col = tmem + lane_base + C::COL_S + sb * C::BN + wg * C::HALF;
-                if constexpr (C::HALF / 2 == 32) {
-                    uint32_t lo[16], hi[16];
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        lo[i] = pk[i];
-                        hi[i] = pk[16 + i];
-                    }
-                    tmem_st16(p_col, lo);
-                    tmem_st16(p_col + 16, hi);
-                } else {
-                    tmem_st16(p_col, *reinterpret_cast<const uint32_t(*)[16]>(pk));
-                }
-                tc::tmem_wait_st();
                 tc::tc_fence_before();
-                tc::mbar_arrive(bar(B_PFULL + sb));
+                tc::mbar_arrive(bar(Bb::PFULL + slot));
             }
             if (!ok) break;
             // ---- epilogue: partial state of this row for this item ----
+            // Every thread waits for the item's O before it frees it, so
+            // arrivals of one item never land in an earlier item's phase.
+            if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::ODONE), uint32_t(k) & 1u, s_abort, P.err,
+                                                       kErrWaitSoftmax))) {
+                ok = false;
+                break;
+            }
+            tc::tc_fence_after();
+            const size_t idx = size_t(it.split) * P.B * P.Hq + size_t(orow);
             if (it.nblk > 0) {
-                if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(B_ODONE + ob), ouse & 1u, s_abort, P.err,
-                                                           kErrWaitSoftmax))) {
-                    ok = false;
-                    break;
-                }
-                tc::tc_fence_after();
-                const size_t idx = size_t(it.split) * P.B * P.Hq + size_t(out_row);
-                float* op = P.ws_o + idx * D + wg * (D / 2);
+                if (rows) {
+                    float* op = P.ws_o + idx * D + wg * C::OCH;
 #pragma unroll
-                for (int q = 0; q < D / 64; ++q) {
-                    float v[32];
-                    tc::tmem_ld32(tmem + lane_base + C::COL_O + ob * D + wg * (D / 2) + q * 32, v);
-                    tc::tmem_wait_ld();
-                    if (valid) {
+                    for (int q = 0; q < C::OCH / 32; ++q) {
+                        float v[32];
+                        tc::tmem_ld32(tmem + lane_base + C::COL_O + wg * C::OCH + q * 32, v);
+                        tc::tmem_wait_ld();
+                        if (valid) {
 #pragma unroll
-                        for (int i = 0; i < 32; i += 4)
-                            *reinterpret_cast<float4*>(op + q * 32 + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+                            for (int i = 0; i < 32; i += 4)
+                                *reinterpret_cast<float4*>(op + q * 32 + i) =
+                                    make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+                        }
                     }
                 }
-                if (wg == 1) xl[row] = l_run;
-                tc::mbar_arrive(bar(B_LXCH));
-                if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(B_LXCH), uint32_t(n_lx) & 1u, s_abort, P.err,
+                // a row's sum is the sum of its two halves' sums
+                float* xb = xl + (k & 1) * (2 * kRows);
+                xb[wg * kRows + row] = l_run;
+                tc::mbar_arrive(bar(Bb::LXCH));
+                if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::LXCH), uint32_t(k) & 1u, s_abort, P.err,
                                                            kErrWaitSoftmax))) {
                     ok = false;
                     break;
                 }
-                ++n_lx;
-                if (wg == 0 && valid) P.ws_ml[idx] = make_float2(m_run, l_run + xl[row]);
-                tc::tc_fence_before();
-                tc::mbar_arrive(bar(B_OFREE + ob));
+                if (wg == 0 && valid) P.ws_ml[idx] = make_float2(m_run, xb[row] + xb[kRows + row]);
             } else {
-                // an empty split: a state with no keys
-                if (wg == 0 && valid) {
-                    const size_t idx = size_t(it.split) * P.B * P.Hq + size_t(out_row);
-                    P.ws_ml[idx] = make_float2(-INFINITY, 0.f);
+                // an empty split: a state with no keys (still one exchange
+                // round, so every item moves the exchange barrier once)
+                tc::mbar_arrive(bar(Bb::LXCH));
+                if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::LXCH), uint32_t(k) & 1u, s_abort, P.err,
+                                                           kErrWaitSoftmax))) {
+                    ok = false;
+                    break;
                 }
-                tc::mbar_arrive(bar(B_OFREE + ob));
-                // matching the MMA side: it commits ODONE for an empty item too
-                tc::mbar_wait(bar(B_ODONE + ob), ouse & 1u, s_abort, P.err, kErrWaitSoftmax);
+                if (wg == 0 && valid) P.ws_ml[idx] = make_float2(-INFINITY, 0.f);
             }
+            tc::tc_fence_before();
+            tc::mbar_arrive(bar(Bb::OFREE));
         }
     }
     tc::tc_fence_before();
     __syncthreads();
     tc::tc_fence_after();
     if (warp == 1) tc::tmem_dealloc(tmem, kTmemCols);
+    // The last CTA to finish resets the work counter for the next launch
+    // (every CTA has claimed its last item before it gets here).
+    if (threadIdx.x == 0) {
+        __threadfence();
+        if (atomicAdd(P.sched + 1, 1u) == gridDim.x - 1) {
+            atomicExch(P.sched, 0u);
+            atomicExch(P.sched + 1, 0u);
+        }
+    }
 }
 
 // cuTensorMapEncodeTiled through the runtime's driver entry point (no -lcuda).
@@ -589,7 +688,7 @@ EncodeFn encode_fn() {
 }
 
 template <int D>
-void launch_d(const TcParams& tp, const CUtensorMap* m, cudaStream_t st) {
+int launch_d(const TcParams& tp, const CUtensorMap* m, cudaStream_t st) {
     static int sms = 0;
     if (!sms) {
         cudaFuncSetAttribute(prefix_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<D>::SMEM);
@@ -599,6 +698,7 @@ void launch_d(const TcParams& tp, const CUtensorMap* m, cudaStream_t st) {
     }
     const unsigned grid = unsigned(tp.n_items < sms ? tp.n_items : sms);
     prefix_tc_kernel<D><<<grid, kThreads, Cfg<D>::SMEM, st>>>(m[0], m[1], m[2], m[3], tp);
+    return 0;
 }
 
 }  // namespace
@@ -618,7 +718,9 @@ int make_kv_tensor_map(void* out_map, const void* base, long rows, int d, int bo
     return r == CUDA_SUCCESS ? 0 : int(cudaErrorInvalidValue);
 }
 
-int prefix_tc_box_rows(int d) { return d == 256 ? Cfg<256>::BN : 128; }
+int prefix_tc_box_rows(int d) {
+    return d == 64 ? Cfg<64>::BN : (d == 128 ? Cfg<128>::BN : Cfg<256>::BN);
+}
 
 int prefix_tc_split_keys(int d, int p_vis, int* nsplit) {
     const int bn = prefix_tc_box_rows(d);
@@ -637,12 +739,14 @@ int launch_prefix_tc(const AttnParams& p, const void* maps, int nsplit, int spli
     const CUtensorMap* m = static_cast<const CUtensorMap*>(maps);
     TcParams tp{p, nsplit, split_keys, p.n_tiles * p.Hkv * nsplit};
     cudaStream_t st = static_cast<cudaStream_t>(stream);
+    int r = int(cudaErrorInvalidValue);
     switch (p.D) {
-        case 64: launch_d<64>(tp, m, st); break;
-        case 128: launch_d<128>(tp, m, st); break;
-        case 256: launch_d<256>(tp, m, st); break;
-        default: return int(cudaErrorInvalidValue);
+        case 64: r = launch_d<64>(tp, m, st); break;
+        case 128: r = launch_d<128>(tp, m, st); break;
+        case 256: r = launch_d<256>(tp, m, st); break;
+        default: break;
     }
+    if (r != 0) return r;
     return int(cudaGetLastError());
 }
 

@@ -79,6 +79,7 @@ struct AttnParams {
     const int32_t* group_src;
     const int32_t* group_seqs;
     unsigned* err;
+    unsigned* sched;              // [2] prompt-span work counter and finished-CTA count, zero between launches
     int B, N, Hq, Hkv, D, G, Tp, T, Dst;
     int layer, step;
     int p_lo, p_hi, s_lo, s_hi;
