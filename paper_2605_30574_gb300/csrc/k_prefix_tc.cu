@@ -9,14 +9,15 @@
 // next item from a launch-wide counter and posts it to the CTA's other roles
 // through a small ring in smem, so CTAs that draw short items take more.
 //
-//   warp 0        TMA producer: claims items; K and V blocks of the item's
-//                 span -> a two-stage smem ring, running ahead across items
+//   warp 0        TMA producer (one lane, two cursors): claims items; K and V
+//                 blocks of the item's span -> two-stage smem rings, each
+//                 block loaded as soon as its stage is free
 //   warp 1        Q K^T issuer (one elected lane): S of the next key block
 //                 into a free TMEM slot (NSLOT slots); owns the TMEM
 //                 allocation
 //   warp 2        Q gather: the tile's query rows -> smem with cp.async,
 //                 one item ahead
-//   warps 3..10   softmax, two warpgroups: each thread owns one row and one
+//   warps 4..11   softmax, two warpgroups: each thread owns one row and one
 //                 half of every block's keys; the halves trade block maxima
 //                 through smem, share one lazily moved reference max, write
 //                 P (bf16) over their own half of the slot in TMEM, rescale
@@ -24,7 +25,7 @@
 //                 end write the row's partial state (m, l, o) to the
 //                 workspace.  Warps whose 32 rows are all past the tile's end
 //                 skip the arithmetic but keep every barrier.
-//   warp 11       P V issuer (one elected lane): O += P V with P read from
+//   warp 3        P V issuer (one elected lane): O += P V with P read from
 //                 TMEM as soon as the softmax has written it -- a separate
 //                 issuer, so P V never queues behind the next Q K^T
 //
@@ -46,8 +47,12 @@ namespace splice {
 namespace {
 
 constexpr int kRows = 128;          // MMA M, rows of one tile
-constexpr int kWarps = 12;          // producer, Q K^T issuer, Q gather, 8 softmax, P V issuer
-constexpr int kPvWarp = 11;
+constexpr int kWarps = 12;          // producer, Q K^T issuer, Q gather, P V issuer, 8 softmax
+constexpr int kPvWarp = 3;
+// Register split (setmaxnreg, per warpgroup): warps 0-3 give registers to
+// the two softmax warpgroups.  256 * 184 + 128 * 112 = 61440 <= the launch's
+// 384 threads * 168.
+constexpr uint32_t kRegsControl = 112, kRegsSoftmax = 184;
 constexpr int kThreads = kWarps * 32;
 constexpr uint32_t kTmemCols = 512;
 constexpr float kTau = 8.0f;        // lazy rescale threshold, log2 units
@@ -56,7 +61,7 @@ constexpr unsigned kErrWaitProducer = 0x1, kErrWaitMma = 0x2, kErrWaitSoftmax = 
                    kErrWaitQ = 0x20, kErrWaitItem = 0x40;
 // Work items reach the CTA's roles through a ring of item numbers in smem.
 constexpr int kItemRing = 8;
-constexpr int kItemTakers = 11;     // Q K^T warp, P V warp, Q gather warp, 8 softmax warps
+constexpr int kItemTakers = 12;     // Q K^T warp, P V warp, Q gather warp, 8 softmax warps, the V cursor
 
 __device__ __forceinline__ float ex2(float x) {
     float y;
@@ -90,34 +95,37 @@ struct Cfg {
     static constexpr int OCH = D / 2;                       // O columns per softmax thread
     static constexpr int KB = D / 64;                       // 64-wide column blocks of Q / K / V
     static constexpr uint32_t KV_BYTES = BN * D * 2;        // one K (or V) block
-    static constexpr int STAGES = int((64u * 1024u) / KV_BYTES);   // 64 KB of K and 64 KB of V in flight
+    // A V block stays in smem from its load until its P V has run, several
+    // blocks later, so V gets the deeper ring: 192 KB of Q, K and V stages.
     static constexpr uint32_t Q_BYTES = kRows * D * 2;      // Q of one tile
-    static constexpr int NQ = (2 * Q_BYTES + 2 * STAGES * KV_BYTES <= 200u * 1024u) ? 2 : 1;   // Q buffers
+    static constexpr int KST = int((64u * 1024u) / KV_BYTES);      // K stages: 64 KB
+    static constexpr int VST = D == 256 ? KST : KST + KST / 2;     // V stages: 96 KB where smem allows
+    static constexpr int NQ = (2 * Q_BYTES + (KST + VST) * KV_BYTES <= 192u * 1024u) ? 2 : 1;   // Q buffers
     // TMEM columns: NSLOT slots of BN columns for S (each softmax thread's
     // P over the first columns of its half of the slot), then O.
     static constexpr int NSLOT = (int(kTmemCols) - D) / BN > 4 ? 4 : (int(kTmemCols) - D) / BN;
     static constexpr uint32_t COL_O = NSLOT * BN;
     static constexpr uint32_t OFF_Q = 0;                    // [NQ] Q buffers
     static constexpr uint32_t OFF_K = OFF_Q + NQ * Q_BYTES;
-    static constexpr uint32_t OFF_V = OFF_K + STAGES * KV_BYTES;
+    static constexpr uint32_t OFF_V = OFF_K + KST * KV_BYTES;
     // exchange: [2 parity][2 half][128] block maxima, [2 parity][2 half][128] row sums
-    static constexpr uint32_t OFF_X = OFF_V + STAGES * KV_BYTES;
+    static constexpr uint32_t OFF_X = OFF_V + VST * KV_BYTES;
     static constexpr uint32_t X_BYTES = 2 * (2 * 2 * kRows) * 4;
     static constexpr uint32_t OFF_BAR = OFF_X + X_BYTES;
     static constexpr uint32_t SMEM = OFF_BAR + 1024 + 1024;   // + barriers, + alignment slack
     static_assert(NSLOT >= 2 && COL_O + D <= kTmemCols, "TMEM budget");
     static_assert(SMEM <= 227 * 1024, "shared memory budget");
-    static_assert(KPT % 32 == 0 && OCH % 32 == 0 && STAGES >= 2, "TMEM access granularity, ring depth");
+    static_assert(KPT % 32 == 0 && OCH % 32 == 0 && VST >= 2, "TMEM access granularity, ring depth");
 };
 
 // Barrier indices (8 bytes each from OFF_BAR).
-template <int STAGES, int NSLOT>
+template <int KST, int VST, int NSLOT>
 struct Bars {
-    static constexpr int KFULL = 0;                       // [STAGES]
-    static constexpr int KEMPTY = STAGES;                 // [STAGES]
-    static constexpr int VFULL = 2 * STAGES;              // [STAGES]
-    static constexpr int VEMPTY = 3 * STAGES;             // [STAGES]
-    static constexpr int SFULL = 4 * STAGES;              // [NSLOT] S computed
+    static constexpr int KFULL = 0;                       // [KST]
+    static constexpr int KEMPTY = KST;                    // [KST]
+    static constexpr int VFULL = 2 * KST;                 // [VST]
+    static constexpr int VEMPTY = 2 * KST + VST;          // [VST]
+    static constexpr int SFULL = 2 * KST + 2 * VST;       // [NSLOT] S computed
     static constexpr int SFREE = SFULL + NSLOT;           // [NSLOT] P of the slot consumed by P V
     static constexpr int PFULL = SFREE + NSLOT;           // [NSLOT] P written (and O rescaled)
     static constexpr int QFULL = PFULL + NSLOT;           // [2]
@@ -125,8 +133,8 @@ struct Bars {
     static constexpr int ODONE = QEMPTY + 2;
     static constexpr int OFREE = ODONE + 1;
     static constexpr int DRAIN = OFREE + 1;               // [issuer]
-    static constexpr int XCH = DRAIN + 2;                 // [2] block-maximum exchange
-    static constexpr int LXCH = XCH + 2;                  // row-sum exchange at an item's end
+    static constexpr int XCH = DRAIN + 2;                 // [2 parity][4 lane quarters] block-maximum exchange
+    static constexpr int LXCH = XCH + 8;                  // row-sum exchange at an item's end
     static constexpr int IFULL = LXCH + 1;                // [kItemRing] item number posted
     static constexpr int IEMPTY = IFULL + kItemRing;      // [kItemRing] item number taken by every role
     static constexpr int COUNT = IEMPTY + kItemRing;
@@ -182,7 +190,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                      const __grid_constant__ CUtensorMap tm_kd, const __grid_constant__ CUtensorMap tm_vd,
                      const TcParams tp) {
     using C = Cfg<D>;
-    using Bb = Bars<C::STAGES, C::NSLOT>;
+    using Bb = Bars<C::KST, C::VST, C::NSLOT>;
     constexpr int NSLOT = C::NSLOT;
     const AttnParams& P = tp.a;
     extern __shared__ uint8_t smem_raw[];
@@ -196,9 +204,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < C::STAGES; ++i) {
+        for (int i = 0; i < C::KST; ++i) {
             tc::mbar_init(bar(Bb::KFULL + i), 1);
             tc::mbar_init(bar(Bb::KEMPTY + i), 1);
+        }
+        for (int i = 0; i < C::VST; ++i) {
             tc::mbar_init(bar(Bb::VFULL + i), 1);
             tc::mbar_init(bar(Bb::VEMPTY + i), 1);
         }
@@ -210,7 +220,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int i = 0; i < 2; ++i) {
             tc::mbar_init(bar(Bb::QFULL + i), 32);
             tc::mbar_init(bar(Bb::QEMPTY + i), 1);
-            tc::mbar_init(bar(Bb::XCH + i), 256);
+            for (int q = 0; q < 4; ++q) tc::mbar_init(bar(Bb::XCH + 4 * i + q), 64);   // the quarter's two warps
             tc::mbar_init(bar(Bb::DRAIN + i), 1);
         }
         tc::mbar_init(bar(Bb::ODONE), 1);
@@ -254,57 +264,125 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto col_s = [](int g) { return uint32_t((g % NSLOT) * C::BN); };
     auto use_of = [](int g) { return uint32_t(g / NSLOT) & 1u; };
 
+    if (warp < 4) {
+    // control warpgroup: give registers to the softmax warpgroups
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsControl));
     if (warp == 0) {
         // ------------------------------------------------ TMA producer
+        // Two cursors in one thread: K blocks are released by Q K^T and V
+        // blocks only later by P V, so each is loaded as soon as its own
+        // stage is free instead of in a fixed K, V, K, V order.  The K
+        // cursor claims items and posts them; the V cursor takes them from
+        // the item ring like the other roles.  Both poll without blocking.
         if (lane == 0) {
-            int jg = 0;          // global block counter of this CTA
-            int issued_k = 0, issued_v = 0;
+            int kpost = 0, vtake = 0;            // items posted / taken by the V cursor
+            int kg = 0, vg = 0;                  // K / V blocks issued (CTA-wide)
+            int kj = 0, vj = 0;                  // block within the cursor's item
+            ItemInfo ki{}, vi{};
+            bool k_in = false, v_in = false, k_done = false, v_done = false;
             int nxt = int(atomicAdd(P.sched, 1u));
-            for (int k = 0; !*s_abort; ++k) {
-                // post the next item to the other roles
-                const int r = k % kItemRing;
-                if (!tc::mbar_wait(bar(Bb::IEMPTY + r), (uint32_t(k / kItemRing) & 1u) ^ 1u, s_abort, P.err,
-                                   kErrWaitProducer))
-                    break;
-                const int item = nxt < tp.n_items ? nxt : -1;
-                s_items[r] = item;
-                tc::mbar_arrive(bar(Bb::IFULL + r));
-                if (item < 0) break;
-                nxt = int(atomicAdd(P.sched, 1u));   // claimed now, needed after this item's copies
-                const ItemInfo it = item_info<D>(P, tp, item);
-                const CUtensorMap* tmk = it.donor ? &tm_kd : &tm_kc;
-                const CUtensorMap* tmv = it.donor ? &tm_vd : &tm_vc;
-                for (int j = 0; j < it.nblk && !*s_abort; ++j, ++jg) {
-                    const int stg = jg % C::STAGES;
-                    const uint32_t use = uint32_t(jg / C::STAGES);
-                    const int y = int(it.span_row + it.k0 + j * C::BN);
-                    if (!tc::mbar_wait(bar(Bb::KEMPTY + stg), (use & 1u) ^ 1u, s_abort, P.err, kErrWaitProducer))
-                        break;
-                    tc::mbar_arrive_expect_tx(bar(Bb::KFULL + stg), C::KV_BYTES);
+            uint64_t idle_since = 0;
+            uint32_t spins = 0;
+            while (!(k_done && v_done)) {
+                bool prog = false;
+                if (!k_done) {
+                    if (!k_in) {
+                        const int r = kpost % kItemRing;
+                        if (tc::mbar_test_wait(bar(Bb::IEMPTY + r), (uint32_t(kpost / kItemRing) & 1u) ^ 1u)) {
+                            const int item = nxt < tp.n_items ? nxt : -1;
+                            s_items[r] = item;
+                            tc::mbar_arrive(bar(Bb::IFULL + r));
+                            ++kpost;
+                            prog = true;
+                            if (item < 0) {
+                                k_done = true;
+                            } else {
+                                nxt = int(atomicAdd(P.sched, 1u));   // claimed now, needed at the next item
+                                ki = item_info<D>(P, tp, item);
+                                kj = 0;
+                                k_in = true;
+                            }
+                        }
+                    }
+                    if (k_in && kj == ki.nblk) k_in = false;
+                    if (k_in) {
+                        const int stg = kg % C::KST;
+                        if (tc::mbar_test_wait(bar(Bb::KEMPTY + stg), (uint32_t(kg / C::KST) & 1u) ^ 1u)) {
+                            const CUtensorMap* tmk = ki.donor ? &tm_kd : &tm_kc;
+                            const int y = int(ki.span_row + ki.k0 + kj * C::BN);
+                            tc::mbar_arrive_expect_tx(bar(Bb::KFULL + stg), C::KV_BYTES);
 #pragma unroll
-                    for (int b = 0; b < C::KB; ++b)
-                        tc::tma_load_2d(sbase + C::OFF_K + stg * C::KV_BYTES + b * (C::BN * 128), tmk, b * 64, y,
-                                        bar(Bb::KFULL + stg));
-                    issued_k = jg + 1;
-                    if (!tc::mbar_wait(bar(Bb::VEMPTY + stg), (use & 1u) ^ 1u, s_abort, P.err, kErrWaitProducer))
-                        break;
-                    tc::mbar_arrive_expect_tx(bar(Bb::VFULL + stg), C::KV_BYTES);
+                            for (int b = 0; b < C::KB; ++b)
+                                tc::tma_load_2d(sbase + C::OFF_K + stg * C::KV_BYTES + b * (C::BN * 128), tmk, b * 64,
+                                                y, bar(Bb::KFULL + stg));
+                            ++kg;
+                            ++kj;
+                            prog = true;
+                        }
+                    }
+                }
+                if (!v_done) {
+                    if (!v_in && vtake < kpost) {
+                        const int r = vtake % kItemRing;
+                        const int item = s_items[r];
+                        tc::mbar_arrive(bar(Bb::IEMPTY + r));
+                        ++vtake;
+                        prog = true;
+                        if (item < 0) {
+                            v_done = true;
+                        } else {
+                            vi = item_info<D>(P, tp, item);
+                            vj = 0;
+                            v_in = true;
+                        }
+                    }
+                    if (v_in && vj == vi.nblk) v_in = false;
+                    if (v_in && vg < kg) {
+                        const int stg = vg % C::VST;
+                        if (tc::mbar_test_wait(bar(Bb::VEMPTY + stg), (uint32_t(vg / C::VST) & 1u) ^ 1u)) {
+                            const CUtensorMap* tmv = vi.donor ? &tm_vd : &tm_vc;
+                            const int y = int(vi.span_row + vi.k0 + vj * C::BN);
+                            tc::mbar_arrive_expect_tx(bar(Bb::VFULL + stg), C::KV_BYTES);
 #pragma unroll
-                    for (int b = 0; b < C::KB; ++b)
-                        tc::tma_load_2d(sbase + C::OFF_V + stg * C::KV_BYTES + b * (C::BN * 128), tmv, b * 64, y,
-                                        bar(Bb::VFULL + stg));
-                    issued_v = jg + 1;
+                            for (int b = 0; b < C::KB; ++b)
+                                tc::tma_load_2d(sbase + C::OFF_V + stg * C::KV_BYTES + b * (C::BN * 128), tmv, b * 64,
+                                                y, bar(Bb::VFULL + stg));
+                            ++vg;
+                            ++vj;
+                            prog = true;
+                        }
+                    }
+                }
+                // bounded: give up after ~1 s without progress, or when another
+                // role did; idle polls back off so they leave the SM's issue
+                // slots to the softmax warps
+                if (prog) {
+                    idle_since = 0;
+                    spins = 0;
+                } else if (++spins > 4) {
+                    __nanosleep(64);
+                }
+                if (!prog && (spins & 63u) == 0) {
+                    if (*s_abort) break;
+                    const uint64_t now = tc::globaltimer_ns();
+                    if (idle_since == 0) {
+                        idle_since = now;
+                    } else if (now - idle_since > 1000000000ull) {
+                        *s_abort = 1;
+                        atomicOr(P.err, kErrWaitProducer);
+                        break;
+                    }
                 }
             }
             // Drain: every issued copy must land before the CTA may exit.
-            for (int j = max(0, issued_k - C::STAGES); j < issued_k; ++j) {
+            for (int j = max(0, kg - C::KST); j < kg; ++j) {
                 volatile int no_abort = 0;
-                tc::mbar_wait(bar(Bb::KFULL + j % C::STAGES), uint32_t(j / C::STAGES) & 1u, &no_abort, P.err,
+                tc::mbar_wait(bar(Bb::KFULL + j % C::KST), uint32_t(j / C::KST) & 1u, &no_abort, P.err,
                               kErrWaitDrain);
             }
-            for (int j = max(0, issued_v - C::STAGES); j < issued_v; ++j) {
+            for (int j = max(0, vg - C::VST); j < vg; ++j) {
                 volatile int no_abort = 0;
-                tc::mbar_wait(bar(Bb::VFULL + j % C::STAGES), uint32_t(j / C::STAGES) & 1u, &no_abort, P.err,
+                tc::mbar_wait(bar(Bb::VFULL + j % C::VST), uint32_t(j / C::VST) & 1u, &no_abort, P.err,
                               kErrWaitDrain);
             }
         }
@@ -331,10 +409,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             }
             for (int j = 0; j < it.nblk; ++j, ++jg) {
-                const int stg = jg % C::STAGES;
+                const int stg = jg % C::KST;
                 const int slot = jg % NSLOT;
                 // the K block is loaded, and the slot's previous P V is done
-                if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::KFULL + stg), uint32_t(jg / C::STAGES) & 1u, s_abort,
+                if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::KFULL + stg), uint32_t(jg / C::KST) & 1u, s_abort,
                                                            P.err, kErrWaitMma)) ||
                     !__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::SFREE + slot), use_of(jg) ^ 1u, s_abort, P.err,
                                                            kErrWaitMma))) {
@@ -379,11 +457,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             const ItemInfo it = item_info<D>(P, tp, item);
             for (int j = 0; j < it.nblk; ++j, ++jg) {
-                const int stg = jg % C::STAGES;
+                const int stg = jg % C::VST;
                 const int slot = jg % NSLOT;
                 if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::PFULL + slot), use_of(jg), s_abort, P.err,
                                                            kErrWaitMma)) ||
-                    !__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::VFULL + stg), uint32_t(jg / C::STAGES) & 1u, s_abort,
+                    !__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::VFULL + stg), uint32_t(jg / C::VST) & 1u, s_abort,
                                                            P.err, kErrWaitMma)) ||
                     (j == 0 && !__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::OFREE), (uint32_t(k) & 1u) ^ 1u, s_abort,
                                                                       P.err, kErrWaitMma)))) {
@@ -446,9 +524,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc::fence_proxy_async_smem();
             tc::mbar_arrive(bar(Bb::QFULL + qb));
         }
+    }
     } else {
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsSoftmax));
         // ------------------------------------------------ softmax / epilogue
-        const int wg = (warp - 3) / 4;                 // 0: first half of each block's keys, 1: second half
+        const int wg = (warp - 4) / 4;                 // 0: first half of each block's keys, 1: second half
         const int quarter = warp & 3;                  // TMEM lane quarter this warp may access
         const int row = quarter * 32 + lane;           // == TMEM lane of this thread's row
         const uint32_t lane_base = uint32_t(quarter * 32) << 16;
@@ -526,12 +606,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                         e0 = fminf(fminf(e0, e1), fminf(e2, e3));
                     }
                 }
-                // the two halves of the block trade their extremes
+                // the two halves of the block trade their extremes (only the
+                // two warps holding this lane quarter's rows meet here)
                 float* xm = xmax + (jg & 1) * (2 * kRows);
                 xm[wg * kRows + row] = e0;
-                tc::mbar_arrive(bar(Bb::XCH + (jg & 1)));
-                if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::XCH + (jg & 1)), uint32_t(jg >> 1) & 1u, s_abort,
-                                                           P.err, kErrWaitSoftmax))) {
+                const uint32_t xch = bar(Bb::XCH + 4 * (jg & 1) + quarter);
+                tc::mbar_arrive(xch);
+                if (!__all_sync(0xffffffffu, tc::mbar_wait(xch, uint32_t(jg >> 1) & 1u, s_abort, P.err, kErrWaitSoftmax))) {
                     ok = false;
                     break;
                 }
