@@ -28,12 +28,14 @@ __global__ void append_kernel(const uint4* __restrict__ kn, const uint4* __restr
 }
 
 // One warp per output row: the partial states of the prompt-span and the
-// generated-span passes (and the ZERO closed form) -> out.
-__global__ void merge_kernel(AttnParams P) {
+// generated-span passes (and the ZERO closed form) -> out.  Rows with up to
+// eight live partials take the one-round-trip path.
+template <int D>
+__global__ void __launch_bounds__(256, 4) merge_kernel(AttnParams P) {
     const long warp = (long(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
     if (warp >= long(P.B) * P.Hq) return;
-    merge_row(P, warp, lane);
+    if (!merge_row_fast<D, 8>(P, warp, lane)) merge_row(P, warp, lane);
 }
 
 }  // namespace
@@ -54,7 +56,14 @@ int launch_merge(const AttnParams& p, void* stream) {
     const long rows = long(p.B) * p.Hq;
     const int block = 256;
     const long threads = rows * 32;
-    merge_kernel<<<unsigned((threads + block - 1) / block), block, 0, static_cast<cudaStream_t>(stream)>>>(p);
+    const unsigned grid = unsigned((threads + block - 1) / block);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    switch (p.D) {
+        case 64: merge_kernel<64><<<grid, block, 0, st>>>(p); break;
+        case 128: merge_kernel<128><<<grid, block, 0, st>>>(p); break;
+        case 256: merge_kernel<256><<<grid, block, 0, st>>>(p); break;
+        default: return int(cudaErrorInvalidValue);
+    }
     return int(cudaGetLastError());
 }
 

@@ -16,32 +16,94 @@
 
 namespace splice {
 
+// Partial slot of the row's i-th live partial: the prompt-span splits first,
+// then the generated-span splits.
+__device__ __forceinline__ int merge_slot(int i, int n_pre) {
+    return i < n_pre ? i : kMaxPrefixSplits + (i - n_pre);
+}
+
+// Lane-parallel weights: lane i < n holds partial i's weight 2^(m_i - M);
+// returns 1 / (sum of weighted row sums), 0 for a row with nothing live.
+__device__ __forceinline__ float merge_weights(const AttnParams& P, long row, int lane, int n, int n_pre,
+                                               bool zero_span, float2 ml, float* w_out) {
+    const float m = ml.x, l = ml.y;
+    float M = (lane < n && l > 0.f) ? m : -INFINITY;
+    if (zero_span) M = fmaxf(M, 0.f);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    const float w = (lane < n && l > 0.f) ? exp2f(m - M) : 0.f;
+    float den = w * l;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) den += __shfl_xor_sync(0xffffffffu, den, off);
+    if (zero_span) den += float(P.p_hi - P.p_lo) * exp2f(0.f - M);
+    *w_out = w;
+    return den > 0.f ? 1.f / den : 0.f;
+}
+
+// Rows with at most NF live partials: every load of the row -- lane i's
+// (m, l) of partial i and this lane's 16-byte slices of o of every partial --
+// is issued before any of them is used, so a row costs one round trip.
+template <int D, int NF>
+__device__ __forceinline__ bool merge_row_fast(const AttnParams& P, long row, int lane) {
+    constexpr int C4 = D / 4;                    // float4 slices of a row
+    constexpr int SL = (C4 + 31) / 32;           // slices per lane
+    const int s = int(row / P.Hq);
+    const uint8_t code = P.src[s];
+    const int n_pre = code == SPLICE_SRC_ZERO ? 0 : P.nsp;
+    const int n = n_pre + P.nss;
+    if (n > NF) return false;
+    const size_t plane = size_t(P.B) * P.Hq;
+    float2 ml = make_float2(-INFINITY, 0.f);
+    if (lane < n) ml = __ldcg(P.ws_ml + size_t(merge_slot(lane, n_pre)) * plane + row);
+    float4 ov[NF][SL];
+#pragma unroll
+    for (int i = 0; i < NF; ++i) {
+        const float4* src = reinterpret_cast<const float4*>(P.ws_o + (size_t(merge_slot(i, n_pre)) * plane + row) * D);
+#pragma unroll
+        for (int q = 0; q < SL; ++q) {
+            const int c = lane + 32 * q;
+            ov[i][q] = (i < n && c < C4) ? __ldcg(src + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+    }
+    float w;
+    const float inv = merge_weights(P, row, lane, n, n_pre, code == SPLICE_SRC_ZERO && P.p_hi > P.p_lo, ml, &w);
+    float4 acc[SL];
+#pragma unroll
+    for (int q = 0; q < SL; ++q) acc[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int i = 0; i < NF; ++i) {
+        const float wi = __shfl_sync(0xffffffffu, w, i);
+        if (i < n && wi != 0.f) {
+#pragma unroll
+            for (int q = 0; q < SL; ++q) {
+                acc[q].x = fmaf(wi, ov[i][q].x, acc[q].x);
+                acc[q].y = fmaf(wi, ov[i][q].y, acc[q].y);
+                acc[q].z = fmaf(wi, ov[i][q].z, acc[q].z);
+                acc[q].w = fmaf(wi, ov[i][q].w, acc[q].w);
+            }
+        }
+    }
+    float4* out = reinterpret_cast<float4*>(P.out + size_t(row) * D);
+#pragma unroll
+    for (int q = 0; q < SL; ++q) {
+        const int c = lane + 32 * q;
+        if (c < C4) out[c] = make_float4(acc[q].x * inv, acc[q].y * inv, acc[q].z * inv, acc[q].w * inv);
+    }
+    return true;
+}
+
+// Any number of live partials (up to kMaxSplits): weights first, then the o
+// slices.
 __device__ __forceinline__ void merge_row(const AttnParams& P, long row, int lane) {
     const int s = int(row / P.Hq);
     const uint8_t code = P.src[s];
     const int n_pre = code == SPLICE_SRC_ZERO ? 0 : P.nsp;
     const int n = n_pre + P.nss;                       // <= kMaxSplits (16)
-    const int p_vis = P.p_hi - P.p_lo;
     const size_t plane = size_t(P.B) * P.Hq;
-    // lane i holds partial i's (m, l), so all of them are in flight at once
-    const int slot = lane < n_pre ? lane : kMaxPrefixSplits + (lane - n_pre);
-    float m = -INFINITY, l = 0.f;
-    if (lane < n) {
-        const float2 ml = __ldcg(P.ws_ml + size_t(slot) * plane + row);
-        m = ml.x;
-        l = ml.y;
-    }
-    const bool zero_span = code == SPLICE_SRC_ZERO && p_vis > 0;
-    float M = l > 0.f ? m : -INFINITY;
-    if (zero_span) M = fmaxf(M, 0.f);
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-    const float w = l > 0.f ? exp2f(m - M) : 0.f;
-    float den = w * l;
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) den += __shfl_xor_sync(0xffffffffu, den, off);
-    if (zero_span) den += float(p_vis) * exp2f(0.f - M);
-    const float inv = den > 0.f ? 1.f / den : 0.f;
+    float2 ml = make_float2(-INFINITY, 0.f);
+    if (lane < n) ml = __ldcg(P.ws_ml + size_t(merge_slot(lane, n_pre)) * plane + row);
+    float w;
+    const float inv = merge_weights(P, row, lane, n, n_pre, code == SPLICE_SRC_ZERO && P.p_hi > P.p_lo, ml, &w);
     float wall[kMaxSplits];
 #pragma unroll
     for (int i = 0; i < kMaxSplits; ++i) wall[i] = __shfl_sync(0xffffffffu, w, i);
@@ -52,8 +114,8 @@ __device__ __forceinline__ void merge_row(const AttnParams& P, long row, int lan
 #pragma unroll
         for (int i = 0; i < kMaxSplits; ++i) {
             if (i < n && wall[i] != 0.f) {
-                const int sl = i < n_pre ? i : kMaxPrefixSplits + (i - n_pre);
-                const float4 o = __ldcg(reinterpret_cast<const float4*>(P.ws_o + (size_t(sl) * plane + row) * P.D) + c);
+                const float4 o = __ldcg(reinterpret_cast<const float4*>(
+                                            P.ws_o + (size_t(merge_slot(i, n_pre)) * plane + row) * P.D) + c);
                 acc.x = fmaf(wall[i], o.x, acc.x);
                 acc.y = fmaf(wall[i], o.y, acc.y);
                 acc.z = fmaf(wall[i], o.z, acc.z);
