@@ -437,6 +437,17 @@ splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const spl
     p.s_chunk = p.nss ? (s_vis + p.nss - 1) / p.nss : 0;
     p.scale_log2 = sh.sm_scale * 1.4426950408889634f;
 
+    // The two passes read disjoint inputs and write disjoint partial slots.
+    // The generated-span pass goes first; the prompt-span pass is queued
+    // right behind it as a programmatic dependent launch, so its CTAs fill
+    // the SMs the generated-span pass's last CTAs leave idle, and it waits
+    // for that pass before it exits.  With per-launch timing on, the events
+    // between the launches serialise them instead.
+    const bool gs_launched = p.nss > 0;
+    if (gs_launched) {
+        e = timed_launch(d, 2, stream, [&] { return splice::launch_generated_span(p, stream); });
+        if (e != cudaSuccess) return cuda_fail(e, "generated-span partials launch");
+    }
     if (p.nsp && p.n_tiles > 0) {
         // Tensor maps over the stores viewed as [rows][d].
         const long rows_c = long(d->P) * sh.num_layers * sh.num_kv_heads * d->Tp;
@@ -449,14 +460,11 @@ splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const spl
                 return fail(SPLICE_ECUDA, "cuTensorMapEncodeTiled failed for store %d", i);
             d->map_ptr[i] = ptrs[i];
         }
+        const bool overlap = gs_launched && !d->profiling;
         e = timed_launch(d, 1, stream, [&] {
-            return splice::launch_prefix_tc(p, d->maps, tc_split, tc_keys, stream);
+            return splice::launch_prefix_tc(p, d->maps, tc_split, tc_keys, stream, overlap);
         });
         if (e != cudaSuccess) return cuda_fail(e, "prompt-span tensor-core pass launch");
-    }
-    if (p.nss) {
-        e = timed_launch(d, 2, stream, [&] { return splice::launch_generated_span(p, stream); });
-        if (e != cudaSuccess) return cuda_fail(e, "generated-span partials launch");
     }
     e = timed_launch(d, 3, stream, [&] { return splice::launch_merge(p, stream); });
     if (e != cudaSuccess) return cuda_fail(e, "merge launch");

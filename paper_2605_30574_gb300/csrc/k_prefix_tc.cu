@@ -739,6 +739,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc::tc_fence_after();
     if (warp == 1) tc::tmem_dealloc(tmem, kTmemCols);
+    // Launched right behind the generated-span pass, this grid may start
+    // while that pass's last CTAs still run (it reads nothing they write);
+    // waiting for it here makes this grid's completion imply that pass's, so
+    // the merge that follows sees both.  A no-op for a plain launch.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     // The last CTA to finish resets the work counter for the next launch
     // (every CTA has claimed its last item before it gets here).
     if (threadIdx.x == 0) {
@@ -769,7 +774,7 @@ EncodeFn encode_fn() {
 }
 
 template <int D>
-int launch_d(const TcParams& tp, const CUtensorMap* m, cudaStream_t st) {
+int launch_d(const TcParams& tp, const CUtensorMap* m, cudaStream_t st, bool overlap_previous) {
     static int sms = 0;
     if (!sms) {
         cudaFuncSetAttribute(prefix_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<D>::SMEM);
@@ -778,8 +783,23 @@ int launch_d(const TcParams& tp, const CUtensorMap* m, cudaStream_t st) {
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     }
     const unsigned grid = unsigned(tp.n_items < sms ? tp.n_items : sms);
-    prefix_tc_kernel<D><<<grid, kThreads, Cfg<D>::SMEM, st>>>(m[0], m[1], m[2], m[3], tp);
-    return 0;
+    if (!overlap_previous) {
+        prefix_tc_kernel<D><<<grid, kThreads, Cfg<D>::SMEM, st>>>(m[0], m[1], m[2], m[3], tp);
+        return 0;
+    }
+    // programmatic dependent launch: CTAs may start as the previous grid's
+    // CTAs retire
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = Cfg<D>::SMEM;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return int(cudaLaunchKernelEx(&cfg, prefix_tc_kernel<D>, m[0], m[1], m[2], m[3], tp));
 }
 
 }  // namespace
@@ -816,15 +836,16 @@ int prefix_tc_split_keys(int d, int p_vis, int* nsplit) {
     return keys;
 }
 
-int launch_prefix_tc(const AttnParams& p, const void* maps, int nsplit, int split_keys, void* stream) {
+int launch_prefix_tc(const AttnParams& p, const void* maps, int nsplit, int split_keys, void* stream,
+                     bool overlap_previous) {
     const CUtensorMap* m = static_cast<const CUtensorMap*>(maps);
     TcParams tp{p, nsplit, split_keys, p.n_tiles * p.Hkv * nsplit};
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     int r = int(cudaErrorInvalidValue);
     switch (p.D) {
-        case 64: r = launch_d<64>(tp, m, st); break;
-        case 128: r = launch_d<128>(tp, m, st); break;
-        case 256: r = launch_d<256>(tp, m, st); break;
+        case 64: r = launch_d<64>(tp, m, st, overlap_previous); break;
+        case 128: r = launch_d<128>(tp, m, st, overlap_previous); break;
+        case 256: r = launch_d<256>(tp, m, st, overlap_previous); break;
         default: break;
     }
     if (r != 0) return r;

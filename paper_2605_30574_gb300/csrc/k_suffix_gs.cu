@@ -104,6 +104,9 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
     using C = GS<D, GT>;
     extern __shared__ __align__(128) uint8_t smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // The prompt-span pass queued behind this grid reads nothing it writes:
+    // let it start as soon as SMs free up.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     uint8_t* ws = smem + warp * C::PER_WARP;
     const uint32_t wbase = tc::smem_u32(ws);
     const uint32_t bar0 = wbase + C::OFF_BAR;

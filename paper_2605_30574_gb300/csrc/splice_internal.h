@@ -106,6 +106,10 @@ int launch_wait_timeout(unsigned* err, unsigned long long limit_ns, void* stream
 int make_kv_tensor_map(void* out_map, const void* base, long rows, int d, int box_rows);
 int prefix_tc_box_rows(int d);
 int prefix_tc_split_keys(int d, int p_vis, int* nsplit);
-int launch_prefix_tc(const AttnParams& p, const void* maps, int nsplit, int split_keys, void* stream);
+// overlap_previous: the launch directly follows the generated-span pass on
+// the same stream and may start while that pass finishes (programmatic
+// dependent launch); the kernel waits for it before it exits.
+int launch_prefix_tc(const AttnParams& p, const void* maps, int nsplit, int split_keys, void* stream,
+                     bool overlap_previous);
 
 }  // namespace splice
