@@ -19,6 +19,9 @@ Legs (one JSON line on rank 0):
 * e2e: the same K steps through the C ABI with the step's queries and new
   K/V copied from pinned host memory and the outputs copied back, copies
   overlapped with compute on separate streams;
+* graph: each timed step's calls (every layer's append and attention)
+  captured once into a CUDA graph before the timed region, then the K graphs
+  replayed under the same events -- the fused-step launch mode;
 * cpu_baseline: the fp64 CPU oracle on a bounded sample of (sequence,
   layer, step) units of the same batch, on the host's cores.
 ``--impl reference`` times that oracle alone as the reference arm.
@@ -327,11 +330,12 @@ def gpu_arm(args):
     outs = torch.empty((N,) + tuple(sb.out.shape), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream()
 
-    def run_step(t, q, k_new, v_new, out):
+    def run_step(t, q, k_new, v_new, out, st=None):
+        st = stream if st is None else st
         for l in range(N):
-            S.suffix_kv_append(sb.desc, l, t, k_new[l], v_new[l], sb.k_suffix, sb.v_suffix, stream)
+            S.suffix_kv_append(sb.desc, l, t, k_new[l], v_new[l], sb.k_suffix, sb.v_suffix, st)
             S.spliced_decode_attn(sb.desc, l, t, q[l], sb.k_clean, sb.v_clean, sb.k_donor, sb.v_donor,
-                                  sb.k_suffix, sb.v_suffix, out[l], sb.ws, stream=stream)
+                                  sb.k_suffix, sb.v_suffix, out[l], sb.ws, stream=st)
 
     for i, t in enumerate(warm):
         run_step(t, wq[i], wkn[i], wvn[i], outs)
@@ -384,6 +388,11 @@ def gpu_arm(args):
                    "GBps": round(per_kind[k] / (v[1] / 1000.0) / 1e9, 1) if v[1] > 0 else None}
                for k, v in prof.items()}
 
+    # ---- graph: every timed step captured once, then replayed ----
+    graph = None
+    if not args.no_graph:
+        graph = graph_leg(sb, steps, qs, kn, vn, outs, run_step, world, dist)
+
     # ---- e2e: host buffers through the C ABI, copies overlapped ----
     e2e = None
     if not args.no_e2e:
@@ -411,12 +420,48 @@ def gpu_arm(args):
                          "bytes_per_launch": per_kind[dom] // max(n_l, 1),
                          "ms_per_launch": ms_l / max(n_l, 1)},
             "kernels": kernels,
-            "e2e": e2e, "gpu_launches": gpu_launches, "clocks": clk.summary(), "cpu_baseline": cpu,
+            "e2e": e2e, "graph": graph, "gpu_launches": gpu_launches, "clocks": clk.summary(),
+            "cpu_baseline": cpu,
         }
         print(json.dumps(line))
     if world > 1:
         dist.destroy_process_group()
     return 0
+
+
+def graph_leg(sb, steps, qs, kn, vn, outs, run_step, world, dist):
+    """The K timed steps, each captured into one CUDA graph (all layers'
+    append + attention) outside the timed region and replayed inside it."""
+    import torch
+    from paper_2605_30574_gb300 import splice as S
+    graphs = []
+    for i, t in enumerate(steps):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            run_step(t, qs[i], kn[i], vn[i], outs, st=torch.cuda.current_stream())
+        graphs.append(g)
+    for g in graphs[:3]:
+        g.replay()
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    ev0.record()
+    for g in graphs:
+        g.replay()
+    ev1.record()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    ms = ev0.elapsed_time(ev1)
+    S.splice_check_device_error(sb.desc)
+    units = sb.B * len(steps)
+    ms, units = reduce_timing(ms, units, dist if world > 1 else None, torch.device("cuda", torch.cuda.current_device()))
+    del graphs
+    return {"value": units / (ms / 1000.0), "unit": UNIT, "ms_per_step": ms / len(steps),
+            "how": "each timed step (all layers: append + attention) captured once into a CUDA graph before "
+                   "the timed region; the K graphs replayed under CUDA events"}
 
 
 def e2e_leg(sb, steps, qs, kn, vn, run_step, dev):
@@ -481,6 +526,7 @@ def main(argv=None):
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--batch", type=int, default=0)
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args(argv)
     if args.impl == "reference":

@@ -1,0 +1,64 @@
+"""A whole decode step -- every layer's generated-span append and spliced
+attention -- captured into one CUDA graph and replayed.
+
+The library's calls must be capture-safe (no synchronisation, no
+allocation; the programmatic dependent launch between the two attention
+passes becomes a graph edge), and a replayed step must give exactly the
+outputs of the same calls issued one by one, replay after replay (the
+prompt-span pass's work counter is reset by its last CTA inside the graph).
+"""
+import pytest
+import torch
+
+from paper_2605_30574_gb300 import build as B
+from paper_2605_30574_gb300.sweep import SweepBatch
+from paper_2605_30574_gb300.synth import workloads as WL
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    B.build()
+
+
+def ladder_slice(layers=6):
+    base = WL.get("qwen3-8b-ladder")
+    Ls = (0, 2, 4, layers)
+    return WL.Workload("ladder-graph", layers, base.num_q_heads, base.num_kv_heads, base.head_dim, 2, 1024,
+                       base.slot_kinds, 400, Ls, base.W_values, base.scaffold_head, base.scaffold_tail, batch=100)
+
+
+@pytest.mark.parametrize("step", [17, 300])
+def test_decode_step_graph_replays_bit_exact(step):
+    wl = ladder_slice()
+    sb = SweepBatch(wl, 0)
+    N = wl.num_layers
+    qs, kns, vns = [], [], []
+    for l in range(N):
+        sb.gen_inputs(l, step)
+        qs.append(sb.q.clone())
+        kns.append(sb.k_new.clone())
+        vns.append(sb.v_new.clone())
+    outs_eager = [torch.empty_like(sb.out) for _ in range(N)]
+    for l in range(N):
+        sb.append(l, step, kns[l], vns[l])
+        sb.attn(l, step, q=qs[l], out=outs_eager[l])
+    torch.cuda.synchronize()
+
+    outs_graph = [torch.full_like(sb.out, float("nan")) for _ in range(N)]
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for l in range(N):
+            sb.append(l, step, kns[l], vns[l])
+            sb.attn(l, step, q=qs[l], out=outs_graph[l])
+    for _ in range(2):
+        for o in outs_graph:
+            o.fill_(float("nan"))
+        g.replay()
+        torch.cuda.synchronize()
+        for l in range(N):
+            assert torch.equal(outs_graph[l], outs_eager[l]), f"layer {l}"
+    from paper_2605_30574_gb300 import splice as S
+    S.splice_check_device_error(sb.desc)
+    sb.close()
