@@ -448,7 +448,8 @@ splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const spl
         e = timed_launch(d, 2, stream, [&] { return splice::launch_generated_span(p, stream); });
         if (e != cudaSuccess) return cuda_fail(e, "generated-span partials launch");
     }
-    if (p.nsp && p.n_tiles > 0) {
+    const bool prefix_launched = p.nsp && p.n_tiles > 0;
+    if (prefix_launched) {
         // Tensor maps over the stores viewed as [rows][d].
         const long rows_c = long(d->P) * sh.num_layers * sh.num_kv_heads * d->Tp;
         const void* ptrs[4] = {k_clean, v_clean, d->Dst ? k_donor : k_clean, d->Dst ? v_donor : v_clean};
@@ -466,7 +467,8 @@ splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const spl
         });
         if (e != cudaSuccess) return cuda_fail(e, "prompt-span tensor-core pass launch");
     }
-    e = timed_launch(d, 3, stream, [&] { return splice::launch_merge(p, stream); });
+    const bool merge_overlap = prefix_launched && !d->profiling;
+    e = timed_launch(d, 3, stream, [&] { return splice::launch_merge(p, stream, merge_overlap); });
     if (e != cudaSuccess) return cuda_fail(e, "merge launch");
     return SPLICE_OK;
 }

@@ -739,6 +739,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc::tc_fence_after();
     if (warp == 1) tc::tmem_dealloc(tmem, kTmemCols);
+    // This CTA's work is done: the merge queued behind this grid may launch
+    // (it waits for the whole grid before it reads anything).  Every CTA of
+    // this grid is running by the time all of them have signalled, so the
+    // merge's CTAs never hold an SM this grid still needs.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     // Launched right behind the generated-span pass, this grid may start
     // while that pass's last CTAs still run (it reads nothing they write);
     // waiting for it here makes this grid's completion imply that pass's, so

@@ -32,6 +32,11 @@ __global__ void append_kernel(const uint4* __restrict__ kn, const uint4* __restr
 // eight live partials take the one-round-trip path.
 template <int D>
 __global__ void __launch_bounds__(256, 4) merge_kernel(AttnParams P) {
+    // Launched behind the prompt-span pass as a programmatic dependent, this
+    // grid may start before that pass has finished: wait for it (and so for
+    // the generated-span pass it waited for) before reading any partial.
+    // A no-op for a plain launch.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     const long warp = (long(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
     if (warp >= long(P.B) * P.Hq) return;
@@ -52,19 +57,25 @@ int launch_append(const uint16_t* kn, const uint16_t* vn, uint16_t* ks, uint16_t
     return int(cudaGetLastError());
 }
 
-int launch_merge(const AttnParams& p, void* stream) {
+int launch_merge(const AttnParams& p, void* stream, bool overlap_previous) {
     const long rows = long(p.B) * p.Hq;
     const int block = 256;
     const long threads = rows * 32;
-    const unsigned grid = unsigned((threads + block - 1) / block);
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(unsigned((threads + block - 1) / block));
+    cfg.blockDim = dim3(block);
+    cfg.stream = static_cast<cudaStream_t>(stream);
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = overlap_previous ? 1 : 0;
     switch (p.D) {
-        case 64: merge_kernel<64><<<grid, block, 0, st>>>(p); break;
-        case 128: merge_kernel<128><<<grid, block, 0, st>>>(p); break;
-        case 256: merge_kernel<256><<<grid, block, 0, st>>>(p); break;
+        case 64: return int(cudaLaunchKernelEx(&cfg, merge_kernel<64>, p));
+        case 128: return int(cudaLaunchKernelEx(&cfg, merge_kernel<128>, p));
+        case 256: return int(cudaLaunchKernelEx(&cfg, merge_kernel<256>, p));
         default: return int(cudaErrorInvalidValue);
     }
-    return int(cudaGetLastError());
 }
 
 }  // namespace splice

@@ -97,7 +97,9 @@ int launch_append(const uint16_t* kn, const uint16_t* vn, uint16_t* ks, uint16_t
                   int N, int Hkv, int D, int T, int layer, int step, void* stream);
 int launch_generated_span(const AttnParams& p, void* stream);
 int generated_span_resident_warps(int d);
-int launch_merge(const AttnParams& p, void* stream);
+// overlap_previous: the launch directly follows the prompt-span pass on the
+// same stream (programmatic dependent launch; the kernel waits for it).
+int launch_merge(const AttnParams& p, void* stream, bool overlap_previous);
 
 // One-thread kernel whose mbarrier wait runs out after limit_ns.
 int launch_wait_timeout(unsigned* err, unsigned long long limit_ns, void* stream);
