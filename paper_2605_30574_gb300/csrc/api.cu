@@ -445,7 +445,7 @@ splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const spl
     // between the launches serialise them instead.
     const bool gs_launched = p.nss > 0;
     if (gs_launched) {
-        e = timed_launch(d, 2, stream, [&] { return splice::launch_generated_span(p, stream); });
+        e = timed_launch(d, 2, stream, [&] { return splice::launch_generated_span(p, stream, !d->profiling); });
         if (e != cudaSuccess) return cuda_fail(e, "generated-span partials launch");
     }
     const bool prefix_launched = p.nsp && p.n_tiles > 0;

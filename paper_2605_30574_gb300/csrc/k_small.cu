@@ -15,6 +15,9 @@ namespace {
 __global__ void append_kernel(const uint4* __restrict__ kn, const uint4* __restrict__ vn,
                               uint4* __restrict__ ks, uint4* __restrict__ vs, int B, int N,
                               int Hkv, int chunks, int T, int layer, int slot) {
+    // the attention call that usually follows may start launching now (it
+    // waits for this grid before it reads anything)
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const long i = long(blockIdx.x) * blockDim.x + threadIdx.x;
     const long total = long(B) * Hkv * chunks;
     if (i >= total) return;

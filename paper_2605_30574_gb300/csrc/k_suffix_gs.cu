@@ -104,6 +104,10 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
     using C = GS<D, GT>;
     extern __shared__ __align__(128) uint8_t smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // Launched as a programmatic dependent of whatever precedes it on the
+    // stream (usually the append of this step's K/V): wait for that grid to
+    // complete before reading anything.  A no-op for a plain launch.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     // The prompt-span pass queued behind this grid reads nothing it writes:
     // let it start as soon as SMs free up.
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -354,7 +358,7 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
 }
 
 template <int D, int GT>
-int launch_gs_t(const AttnParams& p, int n_items, cudaStream_t st) {
+int launch_gs_t(const AttnParams& p, int n_items, cudaStream_t st, bool overlap_previous) {
     using C = GS<D, GT>;
     static int blocks_per_sm = 0, sms = 0;
     if (!blocks_per_sm) {
@@ -367,9 +371,17 @@ int launch_gs_t(const AttnParams& p, int n_items, cudaStream_t st) {
     }
     const long want = (long(n_items) + C::WARPS - 1) / C::WARPS;
     const long cap = long(blocks_per_sm) * sms;
-    const unsigned grid = unsigned(want < cap ? want : cap);
-    gs_kernel<D, GT><<<grid, C::WARPS * 32, C::SMEM, st>>>(p, n_items);
-    return int(cudaGetLastError());
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(unsigned(want < cap ? want : cap));
+    cfg.blockDim = dim3(C::WARPS * 32);
+    cfg.dynamicSmemBytes = C::SMEM;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = overlap_previous ? 1 : 0;
+    return int(cudaLaunchKernelEx(&cfg, gs_kernel<D, GT>, p, n_items));
 }
 
 }  // namespace
@@ -382,21 +394,21 @@ int generated_span_resident_warps(int d) {
     return sms * (d == 256 ? 6 : 8);
 }
 
-int launch_generated_span(const AttnParams& p, void* stream) {
+int launch_generated_span(const AttnParams& p, void* stream, bool overlap_previous) {
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const int gt = p.G % 4 == 0 ? 4 : (p.G % 2 == 0 ? 2 : 1);
     const long n_items = long(p.B) * p.Hkv * (p.G / gt) * p.nss;
     if (n_items == 0) return 0;
     switch (p.D * 8 + gt) {
-        case 64 * 8 + 1: return launch_gs_t<64, 1>(p, int(n_items), st);
-        case 64 * 8 + 2: return launch_gs_t<64, 2>(p, int(n_items), st);
-        case 64 * 8 + 4: return launch_gs_t<64, 4>(p, int(n_items), st);
-        case 128 * 8 + 1: return launch_gs_t<128, 1>(p, int(n_items), st);
-        case 128 * 8 + 2: return launch_gs_t<128, 2>(p, int(n_items), st);
-        case 128 * 8 + 4: return launch_gs_t<128, 4>(p, int(n_items), st);
-        case 256 * 8 + 1: return launch_gs_t<256, 1>(p, int(n_items), st);
-        case 256 * 8 + 2: return launch_gs_t<256, 2>(p, int(n_items), st);
-        case 256 * 8 + 4: return launch_gs_t<256, 4>(p, int(n_items), st);
+        case 64 * 8 + 1: return launch_gs_t<64, 1>(p, int(n_items), st, overlap_previous);
+        case 64 * 8 + 2: return launch_gs_t<64, 2>(p, int(n_items), st, overlap_previous);
+        case 64 * 8 + 4: return launch_gs_t<64, 4>(p, int(n_items), st, overlap_previous);
+        case 128 * 8 + 1: return launch_gs_t<128, 1>(p, int(n_items), st, overlap_previous);
+        case 128 * 8 + 2: return launch_gs_t<128, 2>(p, int(n_items), st, overlap_previous);
+        case 128 * 8 + 4: return launch_gs_t<128, 4>(p, int(n_items), st, overlap_previous);
+        case 256 * 8 + 1: return launch_gs_t<256, 1>(p, int(n_items), st, overlap_previous);
+        case 256 * 8 + 2: return launch_gs_t<256, 2>(p, int(n_items), st, overlap_previous);
+        case 256 * 8 + 4: return launch_gs_t<256, 4>(p, int(n_items), st, overlap_previous);
         default: return int(cudaErrorInvalidValue);
     }
 }

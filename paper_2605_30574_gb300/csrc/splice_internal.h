@@ -95,7 +95,9 @@ void set_last_error(const char* msg);
 // Launchers (return the cudaError_t of the launch as int).
 int launch_append(const uint16_t* kn, const uint16_t* vn, uint16_t* ks, uint16_t* vs, int B,
                   int N, int Hkv, int D, int T, int layer, int step, void* stream);
-int launch_generated_span(const AttnParams& p, void* stream);
+// overlap_previous: launched as a programmatic dependent of the preceding
+// work on the stream (the kernel waits for it before reading anything).
+int launch_generated_span(const AttnParams& p, void* stream, bool overlap_previous);
 int generated_span_resident_warps(int d);
 // overlap_previous: the launch directly follows the prompt-span pass on the
 // same stream (programmatic dependent launch; the kernel waits for it).
