@@ -474,47 +474,55 @@ def e2e_leg(sb, steps, qs, kn, vn, run_step, dev):
     h_q.copy_(qs.cpu())
     h_kn.copy_(kn.cpu())
     h_vn.copy_(vn.cpu())
-    d_q = [torch.empty(qs.shape[1:], dtype=qs.dtype, device=dev) for _ in range(2)]
-    d_kn = [torch.empty(kn.shape[1:], dtype=kn.dtype, device=dev) for _ in range(2)]
-    d_vn = [torch.empty(vn.shape[1:], dtype=vn.dtype, device=dev) for _ in range(2)]
-    d_out = [torch.empty((N,) + tuple(sb.out.shape), dtype=torch.float32, device=dev) for _ in range(2)]
-    h_out = [torch.empty((N,) + tuple(sb.out.shape), dtype=torch.float32, pin_memory=True) for _ in range(2)]
+    # three device slots for inputs and outputs: a copy over the host link
+    # has two compute steps to finish before its slot is needed again
+    NB = 3
+    d_q = [torch.empty(qs.shape[1:], dtype=qs.dtype, device=dev) for _ in range(NB)]
+    d_kn = [torch.empty(kn.shape[1:], dtype=kn.dtype, device=dev) for _ in range(NB)]
+    d_vn = [torch.empty(vn.shape[1:], dtype=vn.dtype, device=dev) for _ in range(NB)]
+    d_out = [torch.empty((N,) + tuple(sb.out.shape), dtype=torch.float32, device=dev) for _ in range(NB)]
+    h_out = [torch.empty((N,) + tuple(sb.out.shape), dtype=torch.float32, pin_memory=True) for _ in range(NB)]
     comp = torch.cuda.current_stream()
     h2d = torch.cuda.Stream()
     d2h = torch.cuda.Stream()
-    in_ready = [torch.cuda.Event() for _ in range(K)]
-    comp_done = [torch.cuda.Event() for _ in range(K)]
-    out_free = [torch.cuda.Event() for _ in range(K)]
-    torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(h2d)
-    for k, t in enumerate(steps):
-        b = k % 2
-        with torch.cuda.stream(h2d):
-            if k >= 2:
-                h2d.wait_event(comp_done[k - 2])          # slot b no longer read by compute
-            d_q[b].copy_(h_q[k], non_blocking=True)
-            d_kn[b].copy_(h_kn[k], non_blocking=True)
-            d_vn[b].copy_(h_vn[k], non_blocking=True)
-            in_ready[k].record(h2d)
-        comp.wait_event(in_ready[k])
-        if k >= 2:
-            comp.wait_event(out_free[k - 2])              # output slot b copied out
-        run_step(t, d_q[b], d_kn[b], d_vn[b], d_out[b])
-        comp_done[k].record(comp)
-        with torch.cuda.stream(d2h):
-            d2h.wait_event(comp_done[k])
-            h_out[b].copy_(d_out[b], non_blocking=True)
-            out_free[k].record(d2h)
-    e1.record(d2h)
-    torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1)
+
+    def pipeline():
+        in_ready = [torch.cuda.Event() for _ in range(K)]
+        comp_done = [torch.cuda.Event() for _ in range(K)]
+        out_free = [torch.cuda.Event() for _ in range(K)]
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(h2d)
+        for k, t in enumerate(steps):
+            b = k % NB
+            with torch.cuda.stream(h2d):
+                if k >= NB:
+                    h2d.wait_event(comp_done[k - NB])         # slot b no longer read by compute
+                d_q[b].copy_(h_q[k], non_blocking=True)
+                d_kn[b].copy_(h_kn[k], non_blocking=True)
+                d_vn[b].copy_(h_vn[k], non_blocking=True)
+                in_ready[k].record(h2d)
+            comp.wait_event(in_ready[k])
+            if k >= NB:
+                comp.wait_event(out_free[k - NB])             # output slot b copied out
+            run_step(t, d_q[b], d_kn[b], d_vn[b], d_out[b])
+            comp_done[k].record(comp)
+            with torch.cuda.stream(d2h):
+                d2h.wait_event(comp_done[k])
+                h_out[b].copy_(d_out[b], non_blocking=True)
+                out_free[k].record(d2h)
+        e1.record(d2h)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1)
+
+    pipeline()          # untimed: first-use costs of the copy path
+    ms = pipeline()
     h2d_bytes = (qs[0].numel() + kn[0].numel() + vn[0].numel()) * 2
     d2h_bytes = d_out[0].numel() * 4
     return {"value": sb.B * K / (ms / 1000.0), "unit": UNIT, "h2d_bytes_per_step": int(h2d_bytes),
             "d2h_bytes_per_step": int(d2h_bytes), "ms_per_step": ms / K,
             "how": "pinned host queries + new K/V per step copied H2D, outputs of every layer copied D2H, "
-                   "on two copy streams overlapped with compute (double-buffered)"}
+                   "on two copy streams overlapped with compute (three device slots)"}
 
 
 def main(argv=None):
