@@ -281,6 +281,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             ItemInfo ki{}, vi{};
             bool k_in = false, v_in = false, k_done = false, v_done = false;
             int nxt = int(atomicAdd(P.sched, 1u));
+            // a span's tiles read it at about the same time; afterwards its
+            // lines go first, keeping the partial states in L2 for the merge
+            const uint64_t pol = tc::l2_policy_evict_first();
             uint64_t idle_since = 0;
             uint32_t spins = 0;
             while (!(k_done && v_done)) {
@@ -313,8 +316,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                             tc::mbar_arrive_expect_tx(bar(Bb::KFULL + stg), C::KV_BYTES);
 #pragma unroll
                             for (int b = 0; b < C::KB; ++b)
-                                tc::tma_load_2d(sbase + C::OFF_K + stg * C::KV_BYTES + b * (C::BN * 128), tmk, b * 64,
-                                                y, bar(Bb::KFULL + stg));
+                                tc::tma_load_2d_hint(sbase + C::OFF_K + stg * C::KV_BYTES + b * (C::BN * 128), tmk, b * 64,
+                                                     y, bar(Bb::KFULL + stg), pol);
                             ++kg;
                             ++kj;
                             prog = true;
@@ -345,8 +348,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                             tc::mbar_arrive_expect_tx(bar(Bb::VFULL + stg), C::KV_BYTES);
 #pragma unroll
                             for (int b = 0; b < C::KB; ++b)
-                                tc::tma_load_2d(sbase + C::OFF_V + stg * C::KV_BYTES + b * (C::BN * 128), tmv, b * 64,
-                                                y, bar(Bb::VFULL + stg));
+                                tc::tma_load_2d_hint(sbase + C::OFF_V + stg * C::KV_BYTES + b * (C::BN * 128), tmv, b * 64,
+                                                     y, bar(Bb::VFULL + stg), pol);
                             ++vg;
                             ++vj;
                             prog = true;

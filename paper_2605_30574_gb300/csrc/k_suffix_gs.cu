@@ -44,10 +44,21 @@ __device__ __forceinline__ float2 unpack2(uint32_t w) {
     return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
 }
 
-__device__ __forceinline__ void bulk_copy(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
-                 "l"(src), "r"(bytes), "r"(bar)
-                 : "memory");
+// Generated-span K/V is read once: the copy marks its L2 lines first to be
+// evicted, so the streamed bytes do not push out the partial states the
+// merge reads right after.
+__device__ __forceinline__ uint64_t l2_evict_first_policy() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+
+__device__ __forceinline__ void bulk_copy(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar, uint64_t pol) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(
+            dst),
+        "l"(src), "r"(bytes), "r"(bar), "l"(pol)
+        : "memory");
 }
 
 template <int D, int GT>
@@ -139,6 +150,7 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
         iss_ok = item_at<D, GT>(P, iss_idx, n_items, iss);
     }
     int issued = 0;
+    const uint64_t pol = l2_evict_first_policy();
     auto issue_next = [&]() {
         if (!iss_ok) return;
         const int stg = issued & 1;
@@ -148,8 +160,8 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
         if (lane == 0) {
             const uint32_t dst = wbase + stg * C::STAGE;
             tc::mbar_arrive_expect_tx(bar0 + 8 * stg, 2 * bytes);
-            bulk_copy(dst, iss.k + size_t(j) * D, bytes, bar0 + 8 * stg);
-            bulk_copy(dst + C::BK * C::ROW, iss.v + size_t(j) * D, bytes, bar0 + 8 * stg);
+            bulk_copy(dst, iss.k + size_t(j) * D, bytes, bar0 + 8 * stg, pol);
+            bulk_copy(dst + C::BK * C::ROW, iss.v + size_t(j) * D, bytes, bar0 + 8 * stg, pol);
         }
         ++issued;
         if (++iss_b >= iss.nblk) {
