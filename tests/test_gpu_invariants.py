@@ -178,3 +178,28 @@ def test_bounded_wait_reports_instead_of_hanging():
     out = a.run(1, 5).clone()                           # the GPU still works
     assert torch.isfinite(out).all()
     S.splice_check_device_error(a.desc)
+
+
+def test_two_descriptors_interleaved_on_one_stream():
+    """Each descriptor carries its own work counters and tables: alternating
+    the calls of two batches on one stream gives exactly the outputs of each
+    batch's calls issued on their own."""
+    wl_a = small_wl()
+    wl_b = WL.Workload("inv2", 4, 8, 2, 128, 2, 300, (WL.BLANK, WL.ZERO), 12, (0, 2), (0, 3), 8, 4,
+                       batch=10 ** 6, seed=5)
+    a = SweepBatch(wl_a, seqs=wl_a.sequences())
+    b = SweepBatch(wl_b, seqs=wl_b.sequences())
+    points = [(l, t) for t in (1, 5, 12) for l in range(4)]
+    alone_a = {p: a.run(*p).clone() for p in points}
+    alone_b = {p: b.run(*p).clone() for p in points}
+    for l, t in points:
+        a.gen_inputs(l, t)
+        b.gen_inputs(l, t)
+        a.append(l, t)
+        b.append(l, t)
+        a.attn(l, t)
+        b.attn(l, t)
+        assert torch.equal(a.out, alone_a[(l, t)]), ("a", l, t)
+        assert torch.equal(b.out, alone_b[(l, t)]), ("b", l, t)
+    S.splice_check_device_error(a.desc)
+    S.splice_check_device_error(b.desc)

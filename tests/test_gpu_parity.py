@@ -227,3 +227,24 @@ def test_full_size_sampled(name):
         a, r = assert_close(g, ref, f"{name} s={s} l={l} t={t}")
         worst = (max(worst[0], a), max(worst[1], r))
     print(name, "points", len(got), "worst abs/rel", worst)
+
+
+# --------------------------------------------------------------------------
+# softmax scale: sign and zero
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("scale", [-0.7, 0.0, 2.5])
+def test_softmax_scale_sign_and_zero(scale):
+    """sm_scale < 0 makes the largest scaled logit the smallest raw one (the
+    kernels then track block minima); 0 gives uniform weights over the visible
+    keys; a large positive scale sharpens the weights so the lazily moved
+    reference max moves more often."""
+    wl = WL.Workload(f"scale{scale}", 3, 8, 2, 128, 2, 300, (WL.BLANK, WL.ZERO, WL.SAME_ALGO), 9,
+                     (0, 1, 3), (0, 2, 10), 4, 2, batch=10 ** 6, sm_scale=scale)
+    sb = SweepBatch(wl, 0)
+    inp = CachedInputs(wl)
+    for t in (1, 2, 9):
+        for l in range(wl.num_layers):
+            out = sb.run(l, t).cpu().numpy()
+            ref = oracle_rows(wl, inp, sb.seqs, l, t, range(sb.B))
+            assert_close(out, ref, f"scale {scale} l={l} t={t}")
+    S.splice_check_device_error(sb.desc)
