@@ -30,6 +30,17 @@ What it computes, step by step, the slow and obvious way:
    standard identity softmax over a union = weighted combination of
    per-part softmaxes; pinned against single-pass softmax in the tests.
 
+5. ``delta_positions`` / ``delta_encode`` / ``delta_decode`` -- the
+   delta encoding of a stored donor span against the clean span of the same
+   prompt, layer and kv head: the positions whose K row or V row differs bit
+   for bit, and the donor rows at those positions in increasing position
+   order.  Table 1's donors are positionally aligned with the clean prompt
+   (§3: scaffolds are trimmed to the same length), so a donor shares every
+   position whose rows are equal; the encoding is lossless by definition
+   (``delta_decode`` rebuilds the donor span exactly), and attention over
+   the donor span is the merge of attention over the clean span without
+   those positions and over the encoded rows (step 4).
+
 Parity is pinned (tests/test_oracle_pins.py) by hand-derived cases
 (tests/golden/), a literal in-place simulation of Algorithm 1, the ZERO
 closed form, torch's CPU scaled_dot_product_attention on materialised
@@ -165,3 +176,38 @@ def merge_partials(parts):
     num = sum(np.exp(m - M) * o for m, _, o in live)
     den = sum(np.exp(m - M) * l for m, l, _ in live)
     return num / den
+
+
+def delta_positions(clean_k, clean_v, donor_k, donor_v) -> np.ndarray:
+    """Positions of one span [T_p][d] (bf16 bit patterns) where the donor
+    differs from the clean span: bool [T_p], True where the K row or the V
+    row is not equal bit for bit."""
+    ck, cv = np.asarray(clean_k, np.uint16), np.asarray(clean_v, np.uint16)
+    dk, dv = np.asarray(donor_k, np.uint16), np.asarray(donor_v, np.uint16)
+    return (ck != dk).any(axis=1) | (cv != dv).any(axis=1)
+
+
+def delta_encode(clean_k, clean_v, donor_k, donor_v):
+    """(mask [T_p] bool, rows_k [n][d], rows_v [n][d]): the differing
+    positions and the donor's rows there, in increasing position order."""
+    mask = delta_positions(clean_k, clean_v, donor_k, donor_v)
+    idx = np.nonzero(mask)[0]
+    return mask, np.asarray(donor_k, np.uint16)[idx].copy(), np.asarray(donor_v, np.uint16)[idx].copy()
+
+
+def delta_decode(clean_k, clean_v, mask, rows_k, rows_v):
+    """The donor span rebuilt from the clean span and its delta encoding."""
+    k = np.array(clean_k, np.uint16, copy=True)
+    v = np.array(clean_v, np.uint16, copy=True)
+    idx = np.nonzero(np.asarray(mask, bool))[0]
+    k[idx] = rows_k
+    v[idx] = rows_v
+    return k, v
+
+
+def pack_mask_words(mask, words: int) -> np.ndarray:
+    """Bit j % 32 of word j // 32 set iff mask[j]; ``words`` uint32 words."""
+    out = np.zeros(words, np.uint32)
+    for j in np.nonzero(np.asarray(mask, bool))[0]:
+        out[j // 32] |= np.uint32(1) << np.uint32(j % 32)
+    return out

@@ -455,3 +455,102 @@ def test_pins_catch_planted_mistakes(monkeypatch):
                     pass
                 m.setattr(so, "attend", lambda q, K, V, lo, s: orig_attend(q, K[:, :-1], V[:, :-1], lo, s))
             assert not _hand_cases_pass(), f"planted mistake '{name}' went unnoticed"
+
+
+# --------------------------------------------------------------------------
+# delta encoding of a donor span against the clean span
+# --------------------------------------------------------------------------
+def test_delta_encoding_hand_case():
+    # T_p = 5, d = 2; bf16 bit patterns.  Position 1 differs in K only,
+    # position 3 in V only, position 4 by the sign of a zero (-0 vs +0 are
+    # different bit patterns, so the position is encoded).
+    one, two, three, neg0 = 0x3F80, 0x4000, 0x4040, 0x8000
+    ck = np.array([[one, two], [one, one], [two, two], [three, 0], [0, one]], np.uint16)
+    cv = np.array([[two, one], [two, two], [one, one], [one, one], [one, 0]], np.uint16)
+    dk = ck.copy()
+    dv = cv.copy()
+    dk[1, 1] = three
+    dv[3, 0] = three
+    dk[4, 0] = neg0
+    mask, rk, rv = oracle.delta_encode(ck, cv, dk, dv)
+    assert mask.tolist() == [False, True, False, True, True]
+    assert rk.tolist() == [[one, three], [three, 0], [neg0, one]]
+    assert rv.tolist() == [[two, two], [three, one], [one, 0]]
+    assert oracle.pack_mask_words(mask, 2).tolist() == [0b11010, 0]
+    bits = np.zeros(64, bool)
+    bits[[0, 31, 32, 63]] = True
+    assert oracle.pack_mask_words(bits, 2).tolist() == [0x80000001, 0x80000001]
+
+
+def test_delta_encoding_round_trip_and_merge_identity():
+    rng = np.random.default_rng(9)
+    for trial in range(20):
+        Tp, d = int(rng.integers(1, 40)), int(rng.integers(1, 6))
+        ck = to_bf16(rng.normal(0, 1, (Tp, d)))
+        cv = to_bf16(rng.normal(0, 1, (Tp, d)))
+        dk, dv = ck.copy(), cv.copy()
+        pick = rng.random(Tp) < rng.random()
+        dk[pick] = to_bf16(rng.normal(0, 1, (int(pick.sum()), d)))
+        vpick = rng.random(Tp) < 0.2
+        dv[vpick] = to_bf16(rng.normal(0, 2, (int(vpick.sum()), d)))
+        mask, rk, rv = oracle.delta_encode(ck, cv, dk, dv)
+        # lossless: the donor span comes back bit for bit
+        bk, bv = oracle.delta_decode(ck, cv, mask, rk, rv)
+        assert np.array_equal(bk, dk) and np.array_equal(bv, dv)
+        # only differing positions are encoded
+        same = ~mask
+        assert np.array_equal(ck[same], dk[same]) and np.array_equal(cv[same], dv[same])
+        # attention over the donor span = merge of the clean span without the
+        # encoded positions and the encoded rows (step 4's identity)
+        q = rng.normal(0, 1, d)
+        K, V = oracle.bf16_to_f64(dk), oracle.bf16_to_f64(dv)
+        want = so.attend(q[None], K[None], V[None], 0, 0.8)[0]
+        got = so.merge_partials([so.partial(q, oracle.bf16_to_f64(ck[same]), oracle.bf16_to_f64(cv[same]), 0.8),
+                                 so.partial(q, oracle.bf16_to_f64(rk), oracle.bf16_to_f64(rv), 0.8)])
+        np.testing.assert_allclose(got, want, rtol=1e-12, atol=1e-13)
+
+
+def test_delta_positions_of_the_ladder_donors():
+    """On the synthetic donor-noise ladder the encoded positions are exactly
+    the perturbed ones (SAME_ALGO / DIFF_ALGO) or every non-scaffold position
+    (BLANK / DIFF_FAMILY), and never a scaffold position."""
+    base = WL.get("qwen3-8b-ladder")
+    wl = WL.Workload("ladder-small", 2, 4, 2, 64, 2, 640, base.slot_kinds, 8, (0, 2), (0, 4),
+                     base.scaffold_head, base.scaffold_tail, batch=40)
+    inp = H.SynthInputs(wl)
+    jj = np.arange(wl.prompt_len)
+    scaffold = (jj < wl.scaffold_head) | (jj >= wl.prompt_len - wl.scaffold_tail)
+    for p in range(2):
+        for k, kind in enumerate(wl.slot_kinds):
+            if kind == WL.ZERO:
+                continue
+            for l in range(wl.num_layers):
+                ck, cv = inp.clean_kv(p, l)
+                dk, dv = inp.donor_kv(p, k, l)
+                for h in range(wl.num_kv_heads):
+                    mask = oracle.delta_positions(ck[h], cv[h], dk[h], dv[h])
+                    assert not mask[scaffold].any()
+                    if kind in (WL.SAME_ALGO, WL.DIFF_ALGO):
+                        assert np.array_equal(mask, inp.perturbed(p, k, jj) & ~scaffold)
+                        frac = mask.sum() / (~scaffold).sum()
+                        want = 0.1 if kind == WL.SAME_ALGO else 0.5
+                        assert abs(frac - want) < 0.08, (kind, frac)
+                    else:
+                        assert mask[~scaffold].all()
+
+
+def test_delta_pins_catch_planted_mistakes(monkeypatch):
+    one, two = 0x3F80, 0x4000
+    ck = np.array([[one], [one]], np.uint16)
+    cv = np.array([[one], [one]], np.uint16)
+    dk = ck.copy()
+    dv = cv.copy()
+    dv[1, 0] = two
+    # a K-only comparison misses position 1
+    with monkeypatch.context() as m:
+        m.setattr(so, "delta_positions", lambda a, b, c, e: (np.asarray(a) != np.asarray(c)).any(axis=1))
+        mask, rk, rv = so.delta_encode(ck, cv, dk, dv)
+        assert not np.array_equal(so.delta_decode(ck, cv, mask, rk, rv)[1], dv)
+    # encoding the clean rows instead of the donor's is caught by the round trip
+    mask = so.delta_positions(ck, cv, dk, dv)
+    assert not np.array_equal(so.delta_decode(ck, cv, mask, ck[mask], cv[mask])[1], dv)
