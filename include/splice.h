@@ -25,7 +25,7 @@
  *     library owns only the descriptor and its device tables.
  *   - `stream` is a cudaStream_t passed as void*; NULL is the legacy default
  *     stream.  Launch calls are asynchronous on that stream and never
- *     synchronise (except splice_debug_source_map and
+ *     synchronise (except splice_debug_source_map, splice_delta_build and
  *     splice_check_device_error, which say so).
  *   - Every call returns a status and never aborts; CUDA errors raised
  *     asynchronously by earlier launches surface as SPLICE_ECUDA on a later
@@ -224,6 +224,83 @@ splice_status spliced_decode_attn_static(splice_desc* desc, int layer, int step,
                                          const splice_bf16* k_donor, const splice_bf16* v_donor,
                                          const splice_bf16* k_suffix, const splice_bf16* v_suffix,
                                          float* out, void* stream);
+
+/*
+ * Delta-donor encoding.  The paper has no counterpart; it changes how a donor
+ * span is read, not what is computed.
+ *
+ * Table 1's donors are aligned position by position with the clean prompt
+ * (§3 trims donor and target prompts to the same length), and a donor may
+ * share many positions with it bit for bit (the synthetic donor-noise
+ * ladder's SAME_ALGO / DIFF_ALGO donors keep 90% / 50% of their content
+ * positions).  Reading such a donor span re-reads bytes that the clean
+ * span's readers read anyway.  The delta encoding of a stored donor span
+ * against the clean span of the same prompt, layer and kv head is the set of
+ * positions whose K row or V row differs bit for bit, as a bitmask, and the
+ * donor's rows at those positions in increasing position order.  It is
+ * lossless, and attention over the donor span equals the log-sum-exp merge
+ * of attention over the clean span without those positions and attention
+ * over the encoded rows.  In delta mode the readers of an encoded slot are
+ * stacked into the clean span's tiles (their encoded positions dropped row
+ * by row) and read the encoded rows as tiles of their own.
+ *
+ * splice_delta_bytes -- bytes of the delta buffer of this descriptor (0 for
+ * NULL or when no slot is stored).  Layout, each part starting on a 256-byte
+ * boundary in this order (W32 = 4 * ceil(prompt_len / 128) words per span):
+ *   mask    [num_prompts][D_stored][N][Hkv][W32] uint32: bit j % 32 of word
+ *           j / 32 set iff position j is encoded
+ *   count   [num_prompts][D_stored][N][Hkv] int32: encoded positions
+ *   rows_k  [num_prompts][D_stored][N][Hkv][prompt_len][d] bf16: rows
+ *           0 .. count-1 hold the encoded donor rows, the rest zeros
+ *   rows_v  same, for V
+ *
+ * splice_delta_build -- encode every stored donor span on `stream`, read the
+ * counts back (this synchronises the stream), and put the descriptor in
+ * delta mode for every stored slot whose encoded fraction (encoded positions
+ * over all positions of the slot's spans) is at most max_fraction; other
+ * slots keep reading the donor store.  slot_fraction (may be NULL) receives
+ * num_donor_slots fractions, -1 for ZERO slots.
+ *   k_clean, v_clean, k_donor, v_donor  the stores later calls will read
+ *   delta         caller-owned device buffer of splice_delta_bytes(desc) bytes
+ *   max_fraction  in [0, 1]
+ * The caller keeps `delta` and the stores' contents unchanged while the
+ * descriptor is in delta mode (encode again after changing a store) and
+ * passes the same stores to spliced_decode_attn.  The descriptor's device
+ * tables are rebuilt: no launch that uses the descriptor may be in flight.
+ * Rejected with SPLICE_EINVAL: a descriptor with a sliding window (the
+ * encoded rows carry no positions), one with no stored slot, or a prompt_len
+ * above 204800.  Outputs of delta mode meet the same tolerance against exact
+ * attention as the default mode but are not bit-identical to it.
+ *
+ * splice_delta_clear -- leave delta mode (device tables rebuilt on `stream`;
+ * no launch that uses the descriptor may be in flight).
+ */
+size_t splice_delta_bytes(const splice_desc* desc);
+splice_status splice_delta_build(splice_desc* desc, const splice_bf16* k_clean, const splice_bf16* v_clean,
+                                 const splice_bf16* k_donor, const splice_bf16* v_donor, void* delta,
+                                 size_t delta_bytes, float max_fraction, float* slot_fraction, void* stream);
+splice_status splice_delta_clear(splice_desc* desc, void* stream);
+
+/*
+ * Planner views for tests (host tables only, no CUDA call).
+ *
+ * splice_debug_plan_delta -- host-only descriptors: re-plan as if the slots
+ * flagged in slot_delta (num_donor_slots bytes; ZERO slots ignored) were in
+ * delta mode.
+ *
+ * splice_debug_plan_rows -- the rows of the prompt-span tiles at (layer,
+ * step), in tile order: out[4 i ..] = (tile, group source, sequence, row
+ * mask), where the group source is SPLICE_SRC_CLEAN, SPLICE_SRC_DONOR0 +
+ * slot, or SPLICE_GROUP_DELTA | (SPLICE_SRC_DONOR0 + slot) for the encoded
+ * rows of a slot, and the row mask is 0 or, for a delta-mode reader in a
+ * clean tile, its stored slot index + 1.  *num_rows receives the count;
+ * with out == NULL only the count is returned, else capacity (in rows) must
+ * cover it.
+ */
+#define SPLICE_GROUP_DELTA 0x100
+splice_status splice_debug_plan_delta(splice_desc* desc, const uint8_t* slot_delta);
+splice_status splice_debug_plan_rows(const splice_desc* desc, int layer, int step, int32_t* out, int capacity,
+                                     int* num_rows);
 
 /*
  * splice_debug_source_map -- the prompt-span source every sequence reads at

@@ -22,6 +22,7 @@ struct splice_desc {
     splice_model_shape shape{};
     int P = 0, Tp = 0, Dslots = 0, Dst = 0, B = 0, T = 0;
     std::vector<int32_t> slot_stored;   // [Dslots] stored-donor index or -1
+    std::vector<splice_donor_kind> kinds;
     std::vector<splice_seq> seqs;
     Plan plan;
     int device = -1;
@@ -36,6 +37,8 @@ struct splice_desc {
     int32_t* d_group_prompt = nullptr;
     int32_t* d_group_src = nullptr;
     int32_t* d_group_seqs = nullptr;
+    int32_t* d_group_mask = nullptr;
+    int32_t* d_slot_delta = nullptr;
     unsigned* d_err = nullptr;
     unsigned* d_sched = nullptr;   // [2] prompt-span work counter, finished-CTA count (zero between launches)
     // Measurement: launch counter and optional per-launch event timing.
@@ -43,10 +46,16 @@ struct splice_desc {
     bool profiling = false;
     std::vector<std::pair<cudaEvent_t, cudaEvent_t>> events[SPLICE_KERNEL_KINDS];
     size_t events_used[SPLICE_KERNEL_KINDS] = {0, 0, 0, 0};
-    // TMA tensor maps of the clean and donor stores (K, V), rebuilt when the
-    // store pointers change.
-    alignas(64) unsigned char maps[4][128] = {};
-    const void* map_ptr[4] = {nullptr, nullptr, nullptr, nullptr};
+    // Delta mode: which slots are read through their delta encoding, the
+    // caller's delta buffer, and the largest encoded count of those slots.
+    std::vector<uint8_t> slot_delta;    // [Dslots]
+    bool delta_on = false;
+    char* delta = nullptr;
+    int delta_max = 0;
+    // TMA tensor maps of the clean and donor stores and of the delta rows
+    // (K, V each), rebuilt when the store pointers change.
+    alignas(64) unsigned char maps[6][128] = {};
+    const void* map_ptr[6] = {nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
 };
 
 namespace {
@@ -143,10 +152,12 @@ splice_status create_common(const splice_model_shape* sh, int P, int Tp, int Dsl
         d->B = B;
         d->T = T;
         d->seqs.assign(seqs, seqs + B);
+        d->kinds.assign(kinds, kinds + Dslots);
+        d->slot_delta.assign(Dslots, 0);
         d->slot_stored.assign(Dslots, -1);
         for (int k = 0; k < Dslots; ++k)
             if (kinds[k] != SPLICE_DONOR_ZERO) d->slot_stored[k] = d->Dst++;
-        std::string e = splice::build_plan(*sh, P, Tp, Dslots, kinds, B, seqs, T, d->plan);
+        std::string e = splice::build_plan(*sh, P, Tp, Dslots, kinds, B, seqs, T, nullptr, d->plan);
         if (!e.empty()) {
             delete d;
             d = nullptr;
@@ -161,6 +172,119 @@ splice_status create_common(const splice_model_shape* sh, int P, int Tp, int Dsl
 }
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// (Re)builds the device table block of a descriptor from its host plan and
+// copies it on `stream`; frees the previous block (no launch that uses it may
+// be in flight).  The error word and the work counter start at zero.
+splice_status upload_tables(splice_desc* d, void* stream) {
+    const Plan& pl = d->plan;
+    struct Part {
+        const void* src;
+        size_t bytes;
+        size_t off;
+    };
+    std::vector<int32_t> seq_prompt(d->B), seq_slot(d->B), slot_delta(d->Dslots);
+    for (int s = 0; s < d->B; ++s) {
+        seq_prompt[s] = d->seqs[s].prompt_id;
+        seq_slot[s] = d->seqs[s].donor_slot;
+    }
+    for (int k = 0; k < d->Dslots; ++k) slot_delta[k] = d->slot_delta[k] ? 1 : 0;
+    const unsigned zero = 0;
+    const unsigned sched_zero[2] = {0, 0};
+    Part parts[] = {
+        {pl.src.data(), pl.src.size(), 0},
+        {seq_prompt.data(), seq_prompt.size() * 4, 0},
+        {seq_slot.data(), seq_slot.size() * 4, 0},
+        {d->slot_stored.data(), d->slot_stored.size() * 4, 0},
+        {pl.tiles.data(), pl.tiles.size() * 4, 0},
+        {pl.group_prompt.data(), pl.group_prompt.size() * 4, 0},
+        {pl.group_src.data(), pl.group_src.size() * 4, 0},
+        {pl.group_seqs.data(), pl.group_seqs.size() * 4, 0},
+        {&zero, sizeof zero, 0},
+        {sched_zero, sizeof sched_zero, 0},
+        {pl.group_mask.data(), pl.group_mask.size() * 4, 0},
+        {slot_delta.data(), slot_delta.size() * 4, 0},
+    };
+    size_t total = 0;
+    for (Part& p : parts) {
+        p.off = total;
+        total = align_up(total + std::max<size_t>(p.bytes, 4), 256);
+    }
+    try {
+        d->staging.assign(total, 0);
+    } catch (const std::bad_alloc&) {
+        return fail(SPLICE_ENOMEM, "host staging allocation failed");
+    }
+    for (const Part& p : parts)
+        if (p.bytes) std::memcpy(d->staging.data() + p.off, p.src, p.bytes);
+    char* b = nullptr;
+    cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&b), total);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return e == cudaErrorMemoryAllocation ? fail(SPLICE_ENOMEM, "cudaMalloc of %zu bytes failed", total)
+                                              : cuda_fail(e, "cudaMalloc");
+    }
+    e = cudaMemcpyAsync(b, d->staging.data(), total, cudaMemcpyHostToDevice, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) {
+        cudaFree(b);
+        return cuda_fail(e, "cudaMemcpyAsync of descriptor tables");
+    }
+    if (d->dev) {
+        e = cudaFree(d->dev);
+        if (e != cudaSuccess) {
+            cudaFree(b);
+            return cuda_fail(e, "cudaFree of the previous descriptor tables");
+        }
+    }
+    d->dev = b;
+    d->d_src = reinterpret_cast<uint8_t*>(b + parts[0].off);
+    d->d_seq_prompt = reinterpret_cast<int32_t*>(b + parts[1].off);
+    d->d_seq_slot = reinterpret_cast<int32_t*>(b + parts[2].off);
+    d->d_slot_stored = reinterpret_cast<int32_t*>(b + parts[3].off);
+    d->d_tiles = reinterpret_cast<int32_t*>(b + parts[4].off);
+    d->d_group_prompt = reinterpret_cast<int32_t*>(b + parts[5].off);
+    d->d_group_src = reinterpret_cast<int32_t*>(b + parts[6].off);
+    d->d_group_seqs = reinterpret_cast<int32_t*>(b + parts[7].off);
+    d->d_err = reinterpret_cast<unsigned*>(b + parts[8].off);
+    d->d_sched = reinterpret_cast<unsigned*>(b + parts[9].off);
+    d->d_group_mask = reinterpret_cast<int32_t*>(b + parts[10].off);
+    d->d_slot_delta = reinterpret_cast<int32_t*>(b + parts[11].off);
+    return SPLICE_OK;
+}
+
+// Layout of the caller's delta buffer (include/splice.h, splice_delta_bytes).
+struct DeltaLayout {
+    size_t spans = 0, mask_off = 0, count_off = 0, k_off = 0, v_off = 0, total = 0;
+    int w32 = 0;
+};
+
+DeltaLayout delta_layout(const splice_desc* d) {
+    DeltaLayout L;
+    if (d->Dst == 0) return L;
+    const splice_model_shape& sh = d->shape;
+    L.spans = size_t(d->P) * d->Dst * sh.num_layers * sh.num_kv_heads;
+    L.w32 = 4 * ((d->Tp + 127) / 128);     // whole 128-key blocks: a tile's last block stays inside
+    const size_t rows = L.spans * size_t(d->Tp) * size_t(sh.head_dim) * 2;
+    L.mask_off = 0;
+    L.count_off = align_up(L.spans * size_t(L.w32) * 4, 256);
+    L.k_off = align_up(L.count_off + L.spans * 4, 256);
+    L.v_off = align_up(L.k_off + rows, 256);
+    L.total = L.v_off + rows;
+    return L;
+}
+
+// Rebuilds the plan for the descriptor's current slot_delta.
+splice_status replan(splice_desc* d) {
+    try {
+        std::string e = splice::build_plan(d->shape, d->P, d->Tp, d->Dslots, d->kinds.data(), d->B, d->seqs.data(), d->T,
+                                           d->slot_delta.data(), d->plan);
+        if (!e.empty()) return fail(SPLICE_EINVAL, "%s", e.c_str());
+    } catch (const std::bad_alloc&) {
+        return fail(SPLICE_ENOMEM, "host allocation failed while planning");
+    }
+    return SPLICE_OK;
+}
+
 
 // Runs one kernel launcher, counting it and, when profiling, bracketing it
 // with a pair of events on its stream.
@@ -240,70 +364,11 @@ splice_status splice_desc_create(const splice_model_shape* sh, int P, int Tp, in
         delete d;
         return cuda_fail(e, "cudaGetDevice");
     }
-    const Plan& pl = d->plan;
-    // Layout of the device table block.
-    struct Part {
-        const void* src;
-        size_t bytes;
-        size_t off;
-    };
-    std::vector<int32_t> seq_prompt(d->B), seq_slot(d->B);
-    for (int s = 0; s < d->B; ++s) {
-        seq_prompt[s] = d->seqs[s].prompt_id;
-        seq_slot[s] = d->seqs[s].donor_slot;
-    }
-    const unsigned zero = 0;
-    const unsigned sched_zero[2] = {0, 0};
-    Part parts[] = {
-        {pl.src.data(), pl.src.size(), 0},
-        {seq_prompt.data(), seq_prompt.size() * 4, 0},
-        {seq_slot.data(), seq_slot.size() * 4, 0},
-        {d->slot_stored.data(), d->slot_stored.size() * 4, 0},
-        {pl.tiles.data(), pl.tiles.size() * 4, 0},
-        {pl.group_prompt.data(), pl.group_prompt.size() * 4, 0},
-        {pl.group_src.data(), pl.group_src.size() * 4, 0},
-        {pl.group_seqs.data(), pl.group_seqs.size() * 4, 0},
-        {&zero, sizeof zero, 0},
-        {sched_zero, sizeof sched_zero, 0},
-    };
-    size_t total = 0;
-    for (Part& p : parts) {
-        p.off = total;
-        total = align_up(total + std::max<size_t>(p.bytes, 4), 256);
-    }
-    try {
-        d->staging.assign(total, 0);
-    } catch (const std::bad_alloc&) {
+    st = upload_tables(d, stream);
+    if (st != SPLICE_OK) {
         delete d;
-        return fail(SPLICE_ENOMEM, "host staging allocation failed");
+        return st;
     }
-    for (const Part& p : parts)
-        if (p.bytes) std::memcpy(d->staging.data() + p.off, p.src, p.bytes);
-    e = cudaMalloc(reinterpret_cast<void**>(&d->dev), total);
-    if (e != cudaSuccess) {
-        cudaGetLastError();
-        delete d;
-        return e == cudaErrorMemoryAllocation ? fail(SPLICE_ENOMEM, "cudaMalloc of %zu bytes failed", total)
-                                              : cuda_fail(e, "cudaMalloc");
-    }
-    e = cudaMemcpyAsync(d->dev, d->staging.data(), total, cudaMemcpyHostToDevice,
-                        static_cast<cudaStream_t>(stream));
-    if (e != cudaSuccess) {
-        cudaFree(d->dev);
-        delete d;
-        return cuda_fail(e, "cudaMemcpyAsync of descriptor tables");
-    }
-    char* b = d->dev;
-    d->d_src = reinterpret_cast<uint8_t*>(b + parts[0].off);
-    d->d_seq_prompt = reinterpret_cast<int32_t*>(b + parts[1].off);
-    d->d_seq_slot = reinterpret_cast<int32_t*>(b + parts[2].off);
-    d->d_slot_stored = reinterpret_cast<int32_t*>(b + parts[3].off);
-    d->d_tiles = reinterpret_cast<int32_t*>(b + parts[4].off);
-    d->d_group_prompt = reinterpret_cast<int32_t*>(b + parts[5].off);
-    d->d_group_src = reinterpret_cast<int32_t*>(b + parts[6].off);
-    d->d_group_seqs = reinterpret_cast<int32_t*>(b + parts[7].off);
-    d->d_err = reinterpret_cast<unsigned*>(b + parts[8].off);
-    d->d_sched = reinterpret_cast<unsigned*>(b + parts[9].off);
     d->on_device = true;
     *out = d;
     return SPLICE_OK;
@@ -418,9 +483,24 @@ splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const spl
     p.s_lo = vis.s_lo;
     p.s_hi = vis.s_hi;
     const int p_vis = vis.p_hi - vis.p_lo, s_vis = vis.s_hi - vis.s_lo;
+    // In delta mode a delta row's span splits and delta-row splits share the
+    // kMaxPrefixSplits prompt-span partial slots.
+    const int max_splits = d->delta_on ? splice::kMaxPrefixSplits / 2 : splice::kMaxPrefixSplits;
     int tc_split = 0, tc_keys = 0;
-    if (p_vis > 0) tc_keys = splice::prefix_tc_split_keys(sh.head_dim, p_vis, &tc_split);
+    if (p_vis > 0) tc_keys = splice::prefix_tc_split_keys(sh.head_dim, p_vis, max_splits, &tc_split);
     p.nsp = tc_split;
+    p.n_span_tiles = d->plan.table_span_tiles[tab];
+    p.group_mask = d->d_group_mask;
+    p.slot_delta = d->d_slot_delta;
+    p.delta_on = d->delta_on ? 1 : 0;
+    p.nsd = 0;
+    if (d->delta_on) {
+        const DeltaLayout dl = delta_layout(d);
+        p.dmask = reinterpret_cast<const uint32_t*>(d->delta + dl.mask_off);
+        p.dcount = reinterpret_cast<const int32_t*>(d->delta + dl.count_off);
+        p.delta_w32 = dl.w32;
+        if (tc_keys > 0) p.nsd = std::min(max_splits, (d->delta_max + tc_keys - 1) / tc_keys);
+    }
     {
         // Generated-span items: (sequence, kv head, row chunk, key split).
         // Split so every resident warp gets about four items, but keep at
@@ -448,14 +528,21 @@ splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const spl
         e = timed_launch(d, 2, stream, [&] { return splice::launch_generated_span(p, stream, !d->profiling); });
         if (e != cudaSuccess) return cuda_fail(e, "generated-span partials launch");
     }
-    const bool prefix_launched = p.nsp && p.n_tiles > 0;
+    const long prefix_items = long(p.n_span_tiles) * sh.num_kv_heads * p.nsp +
+                              long(p.n_tiles - p.n_span_tiles) * sh.num_kv_heads * p.nsd;
+    const bool prefix_launched = p.nsp > 0 && prefix_items > 0;
     if (prefix_launched) {
-        // Tensor maps over the stores viewed as [rows][d].
+        // Tensor maps over the stores viewed as [rows][d]; the delta rows
+        // have the donor store's layout.
         const long rows_c = long(d->P) * sh.num_layers * sh.num_kv_heads * d->Tp;
-        const void* ptrs[4] = {k_clean, v_clean, d->Dst ? k_donor : k_clean, d->Dst ? v_donor : v_clean};
-        const long rows[4] = {rows_c, rows_c, d->Dst ? rows_c * d->Dst : rows_c, d->Dst ? rows_c * d->Dst : rows_c};
+        const long rows_d = d->Dst ? rows_c * d->Dst : rows_c;
+        const DeltaLayout dl = delta_layout(d);
+        const void* xk = d->delta_on ? static_cast<const void*>(d->delta + dl.k_off) : k_clean;
+        const void* xv = d->delta_on ? static_cast<const void*>(d->delta + dl.v_off) : v_clean;
+        const void* ptrs[6] = {k_clean, v_clean, d->Dst ? k_donor : k_clean, d->Dst ? v_donor : v_clean, xk, xv};
+        const long rows[6] = {rows_c, rows_c, rows_d, rows_d, d->delta_on ? rows_d : rows_c, d->delta_on ? rows_d : rows_c};
         const int box = splice::prefix_tc_box_rows(sh.head_dim);
-        for (int i = 0; i < 4; ++i) {
+        for (int i = 0; i < 6; ++i) {
             if (d->map_ptr[i] == ptrs[i]) continue;
             if (splice::make_kv_tensor_map(d->maps[i], ptrs[i], rows[i], sh.head_dim, box) != 0)
                 return fail(SPLICE_ECUDA, "cuTensorMapEncodeTiled failed for store %d", i);
@@ -463,13 +550,140 @@ splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const spl
         }
         const bool overlap = gs_launched && !d->profiling;
         e = timed_launch(d, 1, stream, [&] {
-            return splice::launch_prefix_tc(p, d->maps, tc_split, tc_keys, stream, overlap);
+            return splice::launch_prefix_tc(p, d->maps, tc_keys, stream, overlap);
         });
         if (e != cudaSuccess) return cuda_fail(e, "prompt-span tensor-core pass launch");
     }
     const bool merge_overlap = prefix_launched && !d->profiling;
     e = timed_launch(d, 3, stream, [&] { return splice::launch_merge(p, stream, merge_overlap); });
     if (e != cudaSuccess) return cuda_fail(e, "merge launch");
+    return SPLICE_OK;
+}
+
+size_t splice_delta_bytes(const splice_desc* d) { return d ? delta_layout(d).total : 0; }
+
+splice_status splice_delta_build(splice_desc* d, const splice_bf16* k_clean, const splice_bf16* v_clean,
+                                 const splice_bf16* k_donor, const splice_bf16* v_donor, void* delta,
+                                 size_t delta_bytes, float max_fraction, float* slot_fraction, void* stream) {
+    if (!d) return fail(SPLICE_EINVAL, "descriptor is NULL");
+    if (!d->on_device) return fail(SPLICE_ESTATE, "host-only descriptor");
+    if (d->Dst == 0) return fail(SPLICE_EINVAL, "the descriptor has no stored donor slot");
+    if (d->shape.sliding_window > 0)
+        return fail(SPLICE_EINVAL, "delta encoding needs a descriptor without a sliding window");
+    if (!(max_fraction >= 0.f && max_fraction <= 1.f)) return fail(SPLICE_EINVAL, "max_fraction not in [0, 1]");
+    if (!k_clean || !v_clean || !k_donor || !v_donor || !delta) return fail(SPLICE_EINVAL, "NULL tensor or buffer");
+    const void* ptrs[] = {k_clean, v_clean, k_donor, v_donor, delta};
+    for (const void* p : ptrs)
+        if (!aligned16(p)) return fail(SPLICE_EINVAL, "tensor not 16-byte aligned");
+    const DeltaLayout dl = delta_layout(d);
+    if (delta_bytes < dl.total) return fail(SPLICE_EINVAL, "delta buffer of %zu bytes < %zu", delta_bytes, dl.total);
+    if (size_t(dl.w32) * 8 > 200 * 1024) return fail(SPLICE_EINVAL, "prompt_len %d too long for delta encoding", d->Tp);
+    DeviceGuard g(d->device);
+    if (g.err != cudaSuccess) return cuda_fail(g.err, "cudaSetDevice");
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "earlier CUDA error");
+    const splice_model_shape& sh = d->shape;
+    char* b = static_cast<char*>(delta);
+    e = cudaError_t(splice::launch_delta_build(
+        k_clean, v_clean, k_donor, v_donor, reinterpret_cast<uint32_t*>(b + dl.mask_off),
+        reinterpret_cast<int32_t*>(b + dl.count_off), reinterpret_cast<uint16_t*>(b + dl.k_off),
+        reinterpret_cast<uint16_t*>(b + dl.v_off), d->P, d->Dst, sh.num_layers, sh.num_kv_heads, d->Tp, sh.head_dim,
+        dl.w32, stream));
+    if (e != cudaSuccess) return cuda_fail(e, "delta encoding launch");
+    std::vector<int32_t> counts;
+    try {
+        counts.resize(dl.spans);
+    } catch (const std::bad_alloc&) {
+        return fail(SPLICE_ENOMEM, "host allocation failed");
+    }
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    e = cudaMemcpyAsync(counts.data(), b + dl.count_off, dl.spans * 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(e, "reading the delta counts");
+    // per stored slot: encoded rows / rows of its spans
+    const size_t per_slot = size_t(sh.num_layers) * sh.num_kv_heads;
+    std::vector<double> frac(d->Dst, 0.0);
+    std::vector<int> maxc(d->Dst, 0);
+    for (int p = 0; p < d->P; ++p)
+        for (int stq = 0; stq < d->Dst; ++stq)
+            for (size_t i = 0; i < per_slot; ++i) {
+                const int c = counts[(size_t(p) * d->Dst + stq) * per_slot + i];
+                frac[stq] += c;
+                maxc[stq] = std::max(maxc[stq], c);
+            }
+    const double rows_per_slot = double(d->P) * double(per_slot) * double(d->Tp);
+    std::vector<uint8_t> flags(d->Dslots, 0);
+    int dmax = 0;
+    for (int k = 0; k < d->Dslots; ++k) {
+        const int stq = d->slot_stored[k];
+        const double f = stq < 0 ? -1.0 : frac[stq] / rows_per_slot;
+        if (slot_fraction) slot_fraction[k] = float(f);
+        if (stq >= 0 && f <= double(max_fraction)) {
+            flags[k] = 1;
+            dmax = std::max(dmax, maxc[stq]);
+        }
+    }
+    const std::vector<uint8_t> old_flags = d->slot_delta;
+    d->slot_delta = flags;
+    splice_status s2 = replan(d);
+    if (s2 == SPLICE_OK) s2 = upload_tables(d, stream);
+    if (s2 != SPLICE_OK) {
+        d->slot_delta = old_flags;
+        replan(d);
+        return s2;
+    }
+    d->delta = b;
+    d->delta_max = dmax;
+    d->delta_on = std::any_of(flags.begin(), flags.end(), [](uint8_t f) { return f != 0; });
+    d->map_ptr[4] = d->map_ptr[5] = nullptr;
+    return SPLICE_OK;
+}
+
+splice_status splice_delta_clear(splice_desc* d, void* stream) {
+    if (!d) return fail(SPLICE_EINVAL, "descriptor is NULL");
+    if (!d->on_device) return fail(SPLICE_ESTATE, "host-only descriptor");
+    DeviceGuard g(d->device);
+    if (g.err != cudaSuccess) return cuda_fail(g.err, "cudaSetDevice");
+    std::fill(d->slot_delta.begin(), d->slot_delta.end(), uint8_t(0));
+    splice_status st = replan(d);
+    if (st == SPLICE_OK) st = upload_tables(d, stream);
+    d->delta_on = false;
+    d->delta = nullptr;
+    d->delta_max = 0;
+    d->map_ptr[4] = d->map_ptr[5] = nullptr;
+    return st;
+}
+
+splice_status splice_debug_plan_delta(splice_desc* d, const uint8_t* slot_delta) {
+    if (!d || !slot_delta) return fail(SPLICE_EINVAL, "NULL descriptor or flags");
+    if (d->on_device) return fail(SPLICE_ESTATE, "only host-only descriptors take delta flags without an encoding");
+    for (int k = 0; k < d->Dslots; ++k) d->slot_delta[k] = (slot_delta[k] && d->slot_stored[k] >= 0) ? 1 : 0;
+    return replan(d);
+}
+
+splice_status splice_debug_plan_rows(const splice_desc* d, int layer, int step, int32_t* out, int capacity,
+                                     int* num_rows) {
+    if (!d || !num_rows) return fail(SPLICE_EINVAL, "NULL descriptor or count");
+    if (layer < 0 || layer >= d->shape.num_layers) return fail(SPLICE_EINVAL, "layer %d out of range", layer);
+    if (step < 0 || step > d->T) return fail(SPLICE_EINVAL, "step %d not in [0, %d]", step, d->T);
+    const Plan& pl = d->plan;
+    const int tab = pl.table_of(layer, step);
+    const int t0 = pl.table_tile_off[tab], t1 = pl.table_tile_off[tab + 1];
+    int n = 0;
+    for (int t = t0; t < t1; ++t) n += pl.tiles[4 * size_t(t) + 2];
+    *num_rows = n;
+    if (!out) return SPLICE_OK;
+    if (capacity < n) return fail(SPLICE_EINVAL, "capacity %d < %d rows", capacity, n);
+    int r = 0;
+    for (int t = t0; t < t1; ++t) {
+        const int grp = pl.tiles[4 * size_t(t)], first = pl.tiles[4 * size_t(t) + 1], cnt = pl.tiles[4 * size_t(t) + 2];
+        for (int i = 0; i < cnt; ++i, ++r) {
+            out[4 * size_t(r) + 0] = t - t0;
+            out[4 * size_t(r) + 1] = pl.group_src[grp];
+            out[4 * size_t(r) + 2] = pl.group_seqs[first + i];
+            out[4 * size_t(r) + 3] = pl.group_mask[first + i];
+        }
+    }
     return SPLICE_OK;
 }
 

@@ -29,6 +29,11 @@
 //                 TMEM as soon as the softmax has written it -- a separate
 //                 issuer, so P V never queues behind the next Q K^T
 //
+// Delta mode: a tile of a clean span may hold rows of readers of a
+// delta-encoded donor; for those rows the softmax drops the slot's encoded
+// positions (a per-row bitmask), and items over the slot's encoded rows (a
+// store of their own, split like a span) give the rest of the donor span.
+//
 // The merge kernel combines these partials with those of the generated span
 // (and the ZERO closed form).  Every wait is bounded: a wait that runs out
 // sets a CTA abort flag and an error bit in the descriptor's error word; all
@@ -143,43 +148,69 @@ struct Bars {
 
 struct TcParams {
     AttnParams a;
-    int nsplit;
     int split_keys;     // keys per split (multiple of BN)
+    int n_span_items;   // items [0, n_span_items) read stored spans, the rest delta rows
     int n_items;
 };
 
 // Work item -> tile, kv head, split (consecutive items = consecutive tiles
 // of one (head, split), so a group's tiles read its span at about the same
-// time and share it in L2).
+// time and share it in L2).  Items over stored spans come first, then the
+// items over delta rows (their own split count).
 struct ItemInfo {
-    int h, split, first, nseq, k0, k1, nblk;
+    int h, split, first, nseq, k0, k1, nblk, prompt;
+    int store;          // 0 clean, 1 donor, 2 delta rows
+    bool masked;        // a clean span in delta mode: rows may drop encoded positions
     long span_row;      // first row of the span in the store's 2D view
-    bool donor;
 };
 
 template <int D>
 __device__ __forceinline__ ItemInfo item_info(const AttnParams& P, const TcParams& tp, int item) {
     ItemInfo it;
-    const int tile = item % P.n_tiles;
-    const int hs = item / P.n_tiles;
-    it.split = hs % tp.nsplit;
-    it.h = hs / tp.nsplit;
+    int tile, split;
+    if (item < tp.n_span_items) {
+        tile = item % P.n_span_tiles;
+        const int hs = item / P.n_span_tiles;
+        split = hs % P.nsp;
+        it.h = hs / P.nsp;
+        it.split = split;                      // partial slot
+    } else {
+        const int nd = P.n_tiles - P.n_span_tiles;
+        const int j = item - tp.n_span_items;
+        tile = P.n_span_tiles + j % nd;
+        const int hs = j / nd;
+        split = hs % P.nsd;
+        it.h = hs / P.nsd;
+        it.split = P.nsp + split;              // after the span's own partials
+    }
     const int4 tl = reinterpret_cast<const int4*>(P.tiles)[tile];
     it.first = tl.y;
     it.nseq = tl.z;
-    const int prompt = P.group_prompt[tl.x];
+    it.prompt = P.group_prompt[tl.x];
     const int code = P.group_src[tl.x];
-    it.donor = code != int(SPLICE_SRC_CLEAN);
     long span;
-    if (!it.donor) {
-        span = (long(prompt) * P.N + P.layer) * P.Hkv + it.h;
+    if (code & kGroupDelta) {
+        const int st = P.slot_stored[(code & 0xff) - int(SPLICE_SRC_DONOR0)];
+        span = ((long(it.prompt) * P.Dst + st) * P.N + P.layer) * P.Hkv + it.h;
+        it.store = 2;
+        it.masked = false;
+        it.k0 = split * tp.split_keys;
+        it.k1 = min(P.dcount[span], it.k0 + tp.split_keys);
     } else {
-        const int st = P.slot_stored[code - int(SPLICE_SRC_DONOR0)];
-        span = ((long(prompt) * P.Dst + st) * P.N + P.layer) * P.Hkv + it.h;
+        if (code == int(SPLICE_SRC_CLEAN)) {
+            span = (long(it.prompt) * P.N + P.layer) * P.Hkv + it.h;
+            it.store = 0;
+            it.masked = P.delta_on != 0;
+        } else {
+            const int st = P.slot_stored[code - int(SPLICE_SRC_DONOR0)];
+            span = ((long(it.prompt) * P.Dst + st) * P.N + P.layer) * P.Hkv + it.h;
+            it.store = 1;
+            it.masked = false;
+        }
+        it.k0 = P.p_lo + split * tp.split_keys;
+        it.k1 = min(P.p_hi, it.k0 + tp.split_keys);
     }
     it.span_row = span * P.Tp;
-    it.k0 = P.p_lo + it.split * tp.split_keys;
-    it.k1 = min(P.p_hi, it.k0 + tp.split_keys);
     it.nblk = it.k1 > it.k0 ? (it.k1 - it.k0 + Cfg<D>::BN - 1) / Cfg<D>::BN : 0;
     return it;
 }
@@ -188,6 +219,7 @@ template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     prefix_tc_kernel(const __grid_constant__ CUtensorMap tm_kc, const __grid_constant__ CUtensorMap tm_vc,
                      const __grid_constant__ CUtensorMap tm_kd, const __grid_constant__ CUtensorMap tm_vd,
+                     const __grid_constant__ CUtensorMap tm_kx, const __grid_constant__ CUtensorMap tm_vx,
                      const TcParams tp) {
     using C = Cfg<D>;
     using Bb = Bars<C::KST, C::VST, C::NSLOT>;
@@ -238,6 +270,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc::prefetch_tmap(&tm_vc);
         tc::prefetch_tmap(&tm_kd);
         tc::prefetch_tmap(&tm_vd);
+        if (P.delta_on) {
+            tc::prefetch_tmap(&tm_kx);
+            tc::prefetch_tmap(&tm_vx);
+        }
     }
     if (warp == 1) {
         tc::tmem_alloc(tc::smem_u32(s_tmem), kTmemCols);
@@ -311,7 +347,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (k_in) {
                         const int stg = kg % C::KST;
                         if (tc::mbar_test_wait(bar(Bb::KEMPTY + stg), (uint32_t(kg / C::KST) & 1u) ^ 1u)) {
-                            const CUtensorMap* tmk = ki.donor ? &tm_kd : &tm_kc;
+                            const CUtensorMap* tmk = ki.store == 0 ? &tm_kc : (ki.store == 1 ? &tm_kd : &tm_kx);
                             const int y = int(ki.span_row + ki.k0 + kj * C::BN);
                             tc::mbar_arrive_expect_tx(bar(Bb::KFULL + stg), C::KV_BYTES);
 #pragma unroll
@@ -343,7 +379,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (v_in && vg < kg) {
                         const int stg = vg % C::VST;
                         if (tc::mbar_test_wait(bar(Bb::VEMPTY + stg), (uint32_t(vg / C::VST) & 1u) ^ 1u)) {
-                            const CUtensorMap* tmv = vi.donor ? &tm_vd : &tm_vc;
+                            const CUtensorMap* tmv = vi.store == 0 ? &tm_vc : (vi.store == 1 ? &tm_vd : &tm_vx);
                             const int y = int(vi.span_row + vi.k0 + vj * C::BN);
                             tc::mbar_arrive_expect_tx(bar(Bb::VFULL + stg), C::KV_BYTES);
 #pragma unroll
@@ -459,15 +495,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                 break;
             }
             const ItemInfo it = item_info<D>(P, tp, item);
+            // The softmax has read the previous item's O.  Waited for at every
+            // item, an empty one included, so that ODONE never completes a
+            // second phase before the softmax has seen the first (a parity
+            // wait cannot tell them apart).
+            if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::OFREE), (uint32_t(k) & 1u) ^ 1u, s_abort, P.err,
+                                                       kErrWaitMma))) {
+                ok = false;
+                break;
+            }
             for (int j = 0; j < it.nblk; ++j, ++jg) {
                 const int stg = jg % C::VST;
                 const int slot = jg % NSLOT;
                 if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::PFULL + slot), use_of(jg), s_abort, P.err,
                                                            kErrWaitMma)) ||
                     !__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::VFULL + stg), uint32_t(jg / C::VST) & 1u, s_abort,
-                                                           P.err, kErrWaitMma)) ||
-                    (j == 0 && !__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::OFREE), (uint32_t(k) & 1u) ^ 1u, s_abort,
-                                                                      P.err, kErrWaitMma)))) {
+                                                           P.err, kErrWaitMma))) {
                     ok = false;
                     break;
                 }
@@ -512,7 +555,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::QEMPTY + qb), (quse & 1u) ^ 1u, s_abort, P.err, kErrWaitQ)))
                 break;
             const uint32_t q_s = sbase + C::OFF_Q + qb * C::Q_BYTES;
-            const int nrows = it.nseq * P.G;
+            // an empty split reads no Q
+            const int nrows = it.nblk > 0 ? it.nseq * P.G : 0;
 #pragma unroll 1
             for (int row = lane; row < nrows; row += 32) {
                 const int s = P.group_seqs[it.first + row / P.G];
@@ -539,6 +583,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         float* xl = xmax + 2 * 2 * kRows;                                 // [2][2][128]
         const float c = P.scale_log2;
         const float2 c2 = make_float2(c, c);
+        const float neg = c >= 0.f ? -INFINITY : INFINITY;     // a raw logit that weighs nothing
+        const bool zero_scale = c == 0.f;                      // then neg * c is not -inf
         bool ok = true;
         int jg = 0;
         for (int k = 0;; ++k) {
@@ -556,6 +602,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int s = P.group_seqs[it.first + row / P.G];
                 orow = s * P.Hq + it.h * P.G + row % P.G;
             }
+            // delta mode: the bits of the positions this row's donor
+            // encodes (they come from the delta rows, not from this span)
+            const uint32_t* mrow = nullptr;
+            if (it.masked && valid) {
+                const int mid = P.group_mask[it.first + row / P.G];
+                if (mid > 0)
+                    mrow = P.dmask + size_t(((long(it.prompt) * P.Dst + (mid - 1)) * P.N + P.layer) * P.Hkv + it.h) *
+                                         size_t(P.delta_w32);
+            }
             float m_run = -INFINITY, l_run = 0.f;
             for (int j = 0; j < it.nblk; ++j, ++jg) {
                 const int slot = jg % NSLOT;
@@ -567,9 +622,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 const uint32_t s_col = tmem + lane_base + col_s(jg) + wg * C::KPT;
                 const int kbase = it.k0 + j * C::BN + wg * C::KPT;
-                const bool tail = kbase + C::KPT > it.k1;
                 float s[C::KPT];
                 float e0 = 0.f;
+                // keys of this half that do not count: past the split's end,
+                // and the positions this row's donor encodes
+                uint32_t dead[C::KPT / 32];
+                bool any_dead = false;
                 if (rows) {
                     tc::tc_fence_after();
 #pragma unroll
@@ -579,12 +637,20 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                         for (int i = 0; i < 32; ++i) s[q * 32 + i] = v[i];
                     }
+                    uint32_t anyd = 0u;
+#pragma unroll
+                    for (int q = 0; q < C::KPT / 32; ++q) {
+                        const int live = it.k1 - (kbase + 32 * q);
+                        dead[q] = live >= 32 ? 0u : (live <= 0 ? 0xffffffffu : (0xffffffffu << live));
+                        if (mrow) dead[q] |= __ldg(mrow + (kbase >> 5) + q);
+                        anyd |= dead[q];
+                    }
+                    any_dead = __any_sync(0xffffffffu, anyd != 0u);
                     tc::tmem_wait_ld();
-                    // keys past the split end are masked (only the last block)
-                    if (tail) {
+                    if (any_dead) {
 #pragma unroll
                         for (int i = 0; i < C::KPT; ++i)
-                            if (kbase + i >= it.k1) s[i] = c >= 0.f ? -INFINITY : INFINITY;
+                            if ((dead[i >> 5] >> (i & 31)) & 1u) s[i] = neg;
                     }
                     // extreme of this half's raw logits (max for c >= 0)
                     float e1 = s[1], e2 = s[2], e3 = s[3];
@@ -629,16 +695,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                         resc = j > 0;
                         m_run = mc;
                     }
-                    const float2 nm2 = make_float2(-m_run, -m_run);
+                    // no live key yet (every earlier key of the row dead): any
+                    // finite reference makes the dead keys' weights 0
+                    const float mref = m_run == -INFINITY ? 0.f : m_run;
+                    const float2 nm2 = make_float2(-mref, -mref);
                     float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
                     uint32_t pk[C::KPT / 2];
 #pragma unroll
                     for (int i = 0; i < C::KPT / 2; ++i) {
                         const float2 z = __ffma2_rn(make_float2(s[2 * i], s[2 * i + 1]), c2, nm2);
                         float2 e = make_float2(ex2(z.x), ex2(z.y));
-                        if (tail) {
-                            e.x = kbase + 2 * i < it.k1 ? e.x : 0.f;
-                            e.y = kbase + 2 * i + 1 < it.k1 ? e.y : 0.f;
+                        if (any_dead && zero_scale) {
+                            e.x = ((dead[(2 * i) >> 5] >> ((2 * i) & 31)) & 1u) ? 0.f : e.x;
+                            e.y = ((dead[(2 * i + 1) >> 5] >> ((2 * i + 1) & 31)) & 1u) ? 0.f : e.y;
                         }
                         if (i & 1)
                             acc1 = __fadd2_rn(acc1, e);
@@ -792,7 +861,7 @@ int launch_d(const TcParams& tp, const CUtensorMap* m, cudaStream_t st, bool ove
     }
     const unsigned grid = unsigned(tp.n_items < sms ? tp.n_items : sms);
     if (!overlap_previous) {
-        prefix_tc_kernel<D><<<grid, kThreads, Cfg<D>::SMEM, st>>>(m[0], m[1], m[2], m[3], tp);
+        prefix_tc_kernel<D><<<grid, kThreads, Cfg<D>::SMEM, st>>>(m[0], m[1], m[2], m[3], m[4], m[5], tp);
         return 0;
     }
     // programmatic dependent launch: CTAs may start as the previous grid's
@@ -807,7 +876,7 @@ int launch_d(const TcParams& tp, const CUtensorMap* m, cudaStream_t st, bool ove
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return int(cudaLaunchKernelEx(&cfg, prefix_tc_kernel<D>, m[0], m[1], m[2], m[3], tp));
+    return int(cudaLaunchKernelEx(&cfg, prefix_tc_kernel<D>, m[0], m[1], m[2], m[3], m[4], m[5], tp));
 }
 
 }  // namespace
@@ -831,12 +900,13 @@ int prefix_tc_box_rows(int d) {
     return d == 64 ? Cfg<64>::BN : (d == 128 ? Cfg<128>::BN : Cfg<256>::BN);
 }
 
-int prefix_tc_split_keys(int d, int p_vis, int* nsplit) {
+int prefix_tc_split_keys(int d, int p_vis, int max_splits, int* nsplit) {
     const int bn = prefix_tc_box_rows(d);
-    // Splits depend only on the visible span length, so a row's arithmetic
-    // never depends on which other rows share its tile or launch.
+    // Splits depend only on the visible span length (and the cap), so a
+    // row's arithmetic never depends on which other rows share its tile or
+    // launch.
     int ns = (p_vis + 1023) / 1024;
-    ns = ns < 1 ? 1 : (ns > kMaxPrefixSplits ? kMaxPrefixSplits : ns);
+    ns = ns < 1 ? 1 : (ns > max_splits ? max_splits : ns);
     int keys = (p_vis + ns - 1) / ns;
     keys = (keys + bn - 1) / bn * bn;
     ns = (p_vis + keys - 1) / keys;
@@ -844,10 +914,11 @@ int prefix_tc_split_keys(int d, int p_vis, int* nsplit) {
     return keys;
 }
 
-int launch_prefix_tc(const AttnParams& p, const void* maps, int nsplit, int split_keys, void* stream,
-                     bool overlap_previous) {
+int launch_prefix_tc(const AttnParams& p, const void* maps, int split_keys, void* stream, bool overlap_previous) {
     const CUtensorMap* m = static_cast<const CUtensorMap*>(maps);
-    TcParams tp{p, nsplit, split_keys, p.n_tiles * p.Hkv * nsplit};
+    const int n_span_items = p.n_span_tiles * p.Hkv * p.nsp;
+    TcParams tp{p, split_keys, n_span_items, n_span_items + (p.n_tiles - p.n_span_tiles) * p.Hkv * p.nsd};
+    if (tp.n_items <= 0) return 0;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     int r = int(cudaErrorInvalidValue);
     switch (p.D) {

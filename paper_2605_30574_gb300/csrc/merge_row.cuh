@@ -16,16 +16,32 @@
 
 namespace splice {
 
-// Partial slot of the row's i-th live partial: the prompt-span splits first,
-// then the generated-span splits.
-__device__ __forceinline__ int merge_slot(int i, int n_pre) {
-    return i < n_pre ? i : kMaxPrefixSplits + (i - n_pre);
+// Partials of one row, in merge order: the prompt-span splits, the
+// generated-span splits, then -- a row that reads a delta-encoded donor --
+// its delta-row splits.  Those come last so that a delta row whose delta
+// rows are empty merges exactly as the same row reading the clean span: its
+// extra lanes hold weight 0 where the other row's hold nothing.
+struct RowParts {
+    int span, suffix, delta;
+};
+
+__device__ __forceinline__ RowParts row_parts(const AttnParams& P, uint8_t code) {
+    RowParts r{code == SPLICE_SRC_ZERO ? 0 : P.nsp, P.nss, 0};
+    if (P.delta_on && code >= SPLICE_SRC_DONOR0 && P.slot_delta[code - SPLICE_SRC_DONOR0]) r.delta = P.nsd;
+    return r;
+}
+
+// Workspace slot of the row's i-th partial: prompt-span splits at slots
+// 0.., delta-row splits right after them, generated-span splits from
+// kMaxPrefixSplits on.
+__device__ __forceinline__ int merge_slot(int i, const RowParts& r) {
+    return i < r.span ? i : (i < r.span + r.suffix ? kMaxPrefixSplits + (i - r.span) : i - r.suffix);
 }
 
 // Lane-parallel weights: lane i < n holds partial i's weight 2^(m_i - M);
 // returns 1 / (sum of weighted row sums), 0 for a row with nothing live.
-__device__ __forceinline__ float merge_weights(const AttnParams& P, long row, int lane, int n, int n_pre,
-                                               bool zero_span, float2 ml, float* w_out) {
+__device__ __forceinline__ float merge_weights(const AttnParams& P, int lane, int n, bool zero_span, float2 ml,
+                                               float* w_out) {
     const float m = ml.x, l = ml.y;
     float M = (lane < n && l > 0.f) ? m : -INFINITY;
     if (zero_span) M = fmaxf(M, 0.f);
@@ -49,16 +65,16 @@ __device__ __forceinline__ bool merge_row_fast(const AttnParams& P, long row, in
     constexpr int SL = (C4 + 31) / 32;           // slices per lane
     const int s = int(row / P.Hq);
     const uint8_t code = P.src[s];
-    const int n_pre = code == SPLICE_SRC_ZERO ? 0 : P.nsp;
-    const int n = n_pre + P.nss;
+    const RowParts rp = row_parts(P, code);
+    const int n = rp.span + rp.suffix + rp.delta;
     if (n > NF) return false;
     const size_t plane = size_t(P.B) * P.Hq;
     float2 ml = make_float2(-INFINITY, 0.f);
-    if (lane < n) ml = __ldcg(P.ws_ml + size_t(merge_slot(lane, n_pre)) * plane + row);
+    if (lane < n) ml = __ldcg(P.ws_ml + size_t(merge_slot(lane, rp)) * plane + row);
     float4 ov[NF][SL];
 #pragma unroll
     for (int i = 0; i < NF; ++i) {
-        const float4* src = reinterpret_cast<const float4*>(P.ws_o + (size_t(merge_slot(i, n_pre)) * plane + row) * D);
+        const float4* src = reinterpret_cast<const float4*>(P.ws_o + (size_t(merge_slot(i, rp)) * plane + row) * D);
 #pragma unroll
         for (int q = 0; q < SL; ++q) {
             const int c = lane + 32 * q;
@@ -66,7 +82,7 @@ __device__ __forceinline__ bool merge_row_fast(const AttnParams& P, long row, in
         }
     }
     float w;
-    const float inv = merge_weights(P, row, lane, n, n_pre, code == SPLICE_SRC_ZERO && P.p_hi > P.p_lo, ml, &w);
+    const float inv = merge_weights(P, lane, n, code == SPLICE_SRC_ZERO && P.p_hi > P.p_lo, ml, &w);
     float4 acc[SL];
 #pragma unroll
     for (int q = 0; q < SL; ++q) acc[q] = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -97,13 +113,13 @@ __device__ __forceinline__ bool merge_row_fast(const AttnParams& P, long row, in
 __device__ __forceinline__ void merge_row(const AttnParams& P, long row, int lane) {
     const int s = int(row / P.Hq);
     const uint8_t code = P.src[s];
-    const int n_pre = code == SPLICE_SRC_ZERO ? 0 : P.nsp;
-    const int n = n_pre + P.nss;                       // <= kMaxSplits (16)
+    const RowParts rp = row_parts(P, code);
+    const int n = rp.span + rp.suffix + rp.delta;      // <= kMaxSplits (16)
     const size_t plane = size_t(P.B) * P.Hq;
     float2 ml = make_float2(-INFINITY, 0.f);
-    if (lane < n) ml = __ldcg(P.ws_ml + size_t(merge_slot(lane, n_pre)) * plane + row);
+    if (lane < n) ml = __ldcg(P.ws_ml + size_t(merge_slot(lane, rp)) * plane + row);
     float w;
-    const float inv = merge_weights(P, row, lane, n, n_pre, code == SPLICE_SRC_ZERO && P.p_hi > P.p_lo, ml, &w);
+    const float inv = merge_weights(P, lane, n, code == SPLICE_SRC_ZERO && P.p_hi > P.p_lo, ml, &w);
     float wall[kMaxSplits];
 #pragma unroll
     for (int i = 0; i < kMaxSplits; ++i) wall[i] = __shfl_sync(0xffffffffu, w, i);
@@ -115,7 +131,7 @@ __device__ __forceinline__ void merge_row(const AttnParams& P, long row, int lan
         for (int i = 0; i < kMaxSplits; ++i) {
             if (i < n && wall[i] != 0.f) {
                 const float4 o = __ldcg(reinterpret_cast<const float4*>(
-                                            P.ws_o + (size_t(merge_slot(i, n_pre)) * plane + row) * P.D) + c);
+                                            P.ws_o + (size_t(merge_slot(i, rp)) * plane + row) * P.D) + c);
                 acc.x = fmaf(wall[i], o.x, acc.x);
                 acc.y = fmaf(wall[i], o.y, acc.y);
                 acc.z = fmaf(wall[i], o.z, acc.z);

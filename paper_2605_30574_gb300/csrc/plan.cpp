@@ -9,7 +9,9 @@
 // consecutive distinct W -- inside which every sequence reads one source.
 // One table per rectangle lists that source per sequence and groups the
 // sequences that read the same stored (prompt, source) span, so the prefix
-// pass can read each span once for all its readers.
+// pass can read each span once for all its readers.  In delta mode the
+// readers of a delta-encoded donor slot share the clean span's groups (with
+// a row mask) and read the slot's encoded rows as a group of their own.
 #include <algorithm>
 #include <cstdio>
 #include <numeric>
@@ -34,8 +36,8 @@ static std::string fmt(const char* f, long a = 0, long b = 0) {
     return buf;
 }
 
-std::string build_plan(const splice_model_shape& sh, int P, int Tp, int D, const splice_donor_kind* kinds,
-                       int B, const splice_seq* seqs, int T, Plan& plan) {
+std::string build_plan(const splice_model_shape& sh, int P, int Tp, int Dslots, const splice_donor_kind* kinds,
+                       int B, const splice_seq* seqs, int T, const uint8_t* slot_delta, Plan& plan) {
     const int N = sh.num_layers;
     const int G = sh.num_q_heads / sh.num_kv_heads;
 
@@ -53,18 +55,29 @@ std::string build_plan(const splice_model_shape& sh, int P, int Tp, int D, const
     plan.num_tables = int(eb.size() * cb.size());
     plan.seqs_per_tile = std::max(1, kTileRows / G);
 
+    // stored-donor index of every slot (the non-ZERO slots in slot order)
+    std::vector<int> stored(Dslots, -1);
+    for (int k = 0, n = 0; k < Dslots; ++k)
+        if (kinds[k] != SPLICE_DONOR_ZERO) stored[k] = n++;
+
     plan.src.assign(size_t(plan.num_tables) * B, 0);
     plan.table_group_off.assign(plan.num_tables + 1, 0);
     plan.table_tile_off.assign(plan.num_tables + 1, 0);
+    plan.table_span_tiles.assign(plan.num_tables, 0);
     plan.group_prompt.clear();
     plan.group_src.clear();
     plan.group_first.clear();
     plan.group_count.clear();
     plan.group_seqs.clear();
+    plan.group_mask.clear();
     plan.tiles.clear();
 
-    std::vector<std::tuple<int, int, int>> keyed;   // (prompt, src, seq)
-    keyed.reserve(B);
+    // (delta group?, prompt, group source, row mask, sequence): sorting puts
+    // the stored-span groups first and, inside a group, rows without a mask
+    // first and the rows of each masked slot together.
+    using Key = std::tuple<int, int, int, int, int>;
+    std::vector<Key> keyed;
+    keyed.reserve(2 * size_t(B));
     for (int e = 0; e < int(eb.size()); ++e) {
         for (int c = 0; c < int(cb.size()); ++c) {
             const int tab = e * int(cb.size()) + c;
@@ -79,39 +92,50 @@ std::string build_plan(const splice_model_shape& sh, int P, int Tp, int D, const
                                ? uint8_t(SPLICE_SRC_ZERO)
                                : uint8_t(SPLICE_SRC_DONOR0 + q.donor_slot);
                 src[s] = code;
-                if (code != SPLICE_SRC_ZERO) keyed.emplace_back(q.prompt_id, code, s);
+                if (code == SPLICE_SRC_ZERO) continue;
+                if (code >= SPLICE_SRC_DONOR0 && slot_delta && slot_delta[q.donor_slot]) {
+                    keyed.emplace_back(0, q.prompt_id, int(SPLICE_SRC_CLEAN), stored[q.donor_slot] + 1, s);
+                    keyed.emplace_back(1, q.prompt_id, kGroupDelta | int(code), 0, s);
+                } else {
+                    keyed.emplace_back(0, q.prompt_id, int(code), 0, s);
+                }
             }
             std::sort(keyed.begin(), keyed.end());
             plan.table_group_off[tab] = int(plan.group_prompt.size());
             plan.table_tile_off[tab] = int(plan.tiles.size() / 4);
+            int span_tiles = 0;
             size_t i = 0;
             while (i < keyed.size()) {
                 size_t j = i;
                 while (j < keyed.size() && std::get<0>(keyed[j]) == std::get<0>(keyed[i]) &&
-                       std::get<1>(keyed[j]) == std::get<1>(keyed[i]))
+                       std::get<1>(keyed[j]) == std::get<1>(keyed[i]) && std::get<2>(keyed[j]) == std::get<2>(keyed[i]))
                     ++j;
                 const int gid = int(plan.group_prompt.size());
                 const int first = int(plan.group_seqs.size());
-                plan.group_prompt.push_back(std::get<0>(keyed[i]));
-                plan.group_src.push_back(std::get<1>(keyed[i]));
+                plan.group_prompt.push_back(std::get<1>(keyed[i]));
+                plan.group_src.push_back(std::get<2>(keyed[i]));
                 plan.group_first.push_back(first);
                 plan.group_count.push_back(int(j - i));
-                for (size_t k = i; k < j; ++k) plan.group_seqs.push_back(std::get<2>(keyed[k]));
+                for (size_t k = i; k < j; ++k) {
+                    plan.group_seqs.push_back(std::get<4>(keyed[k]));
+                    plan.group_mask.push_back(std::get<3>(keyed[k]));
+                }
                 for (int off = 0; off < int(j - i); off += plan.seqs_per_tile) {
                     plan.tiles.push_back(gid);
                     plan.tiles.push_back(first + off);
                     plan.tiles.push_back(std::min(plan.seqs_per_tile, int(j - i) - off));
                     plan.tiles.push_back(0);
+                    if (std::get<0>(keyed[i]) == 0) ++span_tiles;
                 }
                 i = j;
             }
+            plan.table_span_tiles[tab] = span_tiles;
         }
     }
     plan.table_group_off[plan.num_tables] = int(plan.group_prompt.size());
     plan.table_tile_off[plan.num_tables] = int(plan.tiles.size() / 4);
     (void)P;
     (void)Tp;
-    (void)D;
     return std::string();
 }
 

@@ -20,6 +20,9 @@ constexpr int kMaxSuffixSplits = 8;
 constexpr int kMaxSplits = kMaxPrefixSplits + kMaxSuffixSplits;
 // Rows of one tensor-core prefix tile (tcgen05 M).
 constexpr int kTileRows = 128;
+// Group source flag: the group reads the delta-encoded rows of a donor slot
+// (group_src = kGroupDelta | (SPLICE_SRC_DONOR0 + slot)).
+constexpr int32_t kGroupDelta = SPLICE_GROUP_DELTA;
 
 // Host-side resolution of the splice rule (§3, Algorithm 1) into tables.
 //
@@ -27,6 +30,13 @@ constexpr int kTileRows = 128;
 // are 0 and every distinct W <= max_steps; layer class c covers layers
 // [class_bounds[c], class_bounds[c+1]) with bounds 0 and every distinct
 // L < N.  Within one (epoch, class) pair every sequence reads one source.
+//
+// Delta mode (a slot flagged in slot_delta): a reader of that slot's donor
+// joins the (prompt, CLEAN) group with row mask = its stored slot index + 1
+// (the prompt-span pass drops the slot's encoded positions from the clean
+// span for its rows) and also forms a (prompt, kGroupDelta | source) group
+// over the slot's encoded rows.  Groups of stored spans come first in every
+// table, delta groups after them.
 struct Plan {
     std::vector<int> epoch_bounds;
     std::vector<int> class_bounds;
@@ -39,17 +49,21 @@ struct Plan {
     std::vector<int32_t> group_first;       // [groups] offset into group_seqs
     std::vector<int32_t> group_count;       // [groups]
     std::vector<int32_t> group_seqs;        // concatenated sequence indices
+    std::vector<int32_t> group_mask;        // parallel to group_seqs: 0, or stored slot + 1 (delta rows)
     // Row tiles of at most kTileRows rows (seqs_per_tile sequences x G heads).
     std::vector<int32_t> table_tile_off;    // [num_tables + 1]
     std::vector<int32_t> tiles;             // [tiles][4]: group, first, count, 0
+    std::vector<int32_t> table_span_tiles;  // [num_tables] tiles of stored-span groups (the rest read delta rows)
     int seqs_per_tile = 0;
 
     int table_of(int layer, int step) const;
 };
 
+// slot_delta: [num_donor_slots] nonzero = the slot is read in delta mode
+// (NULL = no slot).
 std::string build_plan(const splice_model_shape& shape, int num_prompts, int prompt_len,
                        int num_donor_slots, const splice_donor_kind* kinds, int num_seqs,
-                       const splice_seq* seqs, int max_steps, Plan& plan);
+                       const splice_seq* seqs, int max_steps, const uint8_t* slot_delta, Plan& plan);
 
 // Visible key ranges of the step-t query at layer l: prompt positions
 // [p_lo, prompt_len) and generated entries [s_lo, step).
@@ -78,14 +92,22 @@ struct AttnParams {
     const int32_t* group_prompt;
     const int32_t* group_src;
     const int32_t* group_seqs;
+    // delta mode (delta_on != 0)
+    const int32_t* group_mask;    // parallel to group_seqs
+    const uint32_t* dmask;        // [P][Dst][N][Hkv][delta_w32] encoded-position bits
+    const int32_t* dcount;        // [P][Dst][N][Hkv] encoded rows per span
+    const int32_t* slot_delta;    // [num_slots] 1 = the slot is read in delta mode
     unsigned* err;
     unsigned* sched;              // [2] prompt-span work counter and finished-CTA count, zero between launches
     int B, N, Hq, Hkv, D, G, Tp, T, Dst;
     int layer, step;
     int p_lo, p_hi, s_lo, s_hi;
     int nsp, nss;                 // splits of the prompt span / generated span
+    int nsd;                      // splits of the delta rows (delta mode)
+    int delta_on, delta_w32;
     int p_chunk, s_chunk;         // keys per split
     int n_tiles;
+    int n_span_tiles;             // tiles [0, n_span_tiles) read stored spans, the rest delta rows
     float scale_log2;             // sm_scale * log2(e)
 };
 
@@ -109,11 +131,21 @@ int launch_wait_timeout(unsigned* err, unsigned long long limit_ns, void* stream
 // Tensor-core prompt-span pass.  A tensor map is a 128-byte CUtensorMap.
 int make_kv_tensor_map(void* out_map, const void* base, long rows, int d, int box_rows);
 int prefix_tc_box_rows(int d);
-int prefix_tc_split_keys(int d, int p_vis, int* nsplit);
+// Keys per split of a visible span of p_vis keys and the number of splits
+// (at most max_splits).
+int prefix_tc_split_keys(int d, int p_vis, int max_splits, int* nsplit);
+// maps: six tensor maps -- clean K, V; donor K, V; delta rows K, V.
 // overlap_previous: the launch directly follows the generated-span pass on
 // the same stream and may start while that pass finishes (programmatic
 // dependent launch); the kernel waits for it before it exits.
-int launch_prefix_tc(const AttnParams& p, const void* maps, int nsplit, int split_keys, void* stream,
-                     bool overlap_previous);
+int launch_prefix_tc(const AttnParams& p, const void* maps, int split_keys, void* stream, bool overlap_previous);
+
+// Delta encoding of every stored donor span (one CTA per span): bits of the
+// positions whose K or V row differs from the clean span, their count, and
+// the donor rows at those positions compacted to the front of the span's
+// rows in the delta store (the remaining rows zeroed).
+int launch_delta_build(const uint16_t* kc, const uint16_t* vc, const uint16_t* kd, const uint16_t* vd,
+                       uint32_t* mask, int32_t* count, uint16_t* xk, uint16_t* xv, int P, int Dst, int N,
+                       int Hkv, int Tp, int D, int w32, void* stream);
 
 }  // namespace splice

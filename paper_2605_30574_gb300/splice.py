@@ -58,6 +58,13 @@ SIGNATURES = {
     "splice_debug_source_map": (_c_int, [_vp, _c_int, _c_int, ctypes.POINTER(ctypes.c_uint8)]),
     "splice_plan_stats": (_c_int, [_vp, _c_int, _c_int, ctypes.POINTER(_c_int), ctypes.POINTER(_c_int),
                                    ctypes.POINTER(_c_int), ctypes.POINTER(_c_int)]),
+    "splice_delta_bytes": (ctypes.c_size_t, [_vp]),
+    "splice_delta_build": (_c_int, [_vp, _vp, _vp, _vp, _vp, _vp, ctypes.c_size_t, ctypes.c_float,
+                                    ctypes.POINTER(ctypes.c_float), _vp]),
+    "splice_delta_clear": (_c_int, [_vp, _vp]),
+    "splice_debug_plan_delta": (_c_int, [_vp, ctypes.POINTER(ctypes.c_uint8)]),
+    "splice_debug_plan_rows": (_c_int, [_vp, _c_int, _c_int, ctypes.POINTER(ctypes.c_int32), _c_int,
+                                        ctypes.POINTER(_c_int)]),
     "splice_check_device_error": (_c_int, [_vp]),
     "splice_debug_wait_timeout": (_c_int, [_vp, ctypes.c_uint, _vp]),
     "splice_kernel_launches": (ctypes.c_longlong, [_vp]),
@@ -118,10 +125,11 @@ def _stream(stream):
 class Desc:
     """Owns a ``splice_desc*``; destroyed on ``close()`` or garbage collection."""
 
-    def __init__(self, handle: int, num_seqs: int, on_device: bool):
+    def __init__(self, handle: int, num_seqs: int, on_device: bool, slot_kinds=()):
         self.handle = handle
         self.num_seqs = num_seqs
         self.on_device = on_device
+        self.slot_kinds = tuple(int(k) for k in slot_kinds)
 
     def close(self):
         if self.handle:
@@ -134,6 +142,10 @@ class Desc:
                 lib().splice_desc_destroy(self.handle)
         except Exception:
             pass
+
+
+def _desc_slots(desc: Desc):
+    return desc.slot_kinds
 
 
 def _marshal(shape, slot_kinds, seqs):
@@ -151,7 +163,7 @@ def splice_desc_create(shape, num_prompts, prompt_len, slot_kinds, seqs, max_ste
     _check(lib().splice_desc_create(ctypes.byref(sh), num_prompts, prompt_len, len(slot_kinds), kinds,
                                     len(seqs), arr, max_steps, _stream(stream), ctypes.byref(out)),
            "splice_desc_create")
-    return Desc(out.value, len(seqs), True)
+    return Desc(out.value, len(seqs), True, slot_kinds)
 
 
 def splice_desc_create_host(shape, num_prompts, prompt_len, slot_kinds, seqs, max_steps) -> Desc:
@@ -161,7 +173,7 @@ def splice_desc_create_host(shape, num_prompts, prompt_len, slot_kinds, seqs, ma
     _check(lib().splice_desc_create_host(ctypes.byref(sh), num_prompts, prompt_len, len(slot_kinds), kinds,
                                          len(seqs), arr, max_steps, ctypes.byref(out)),
            "splice_desc_create_host")
-    return Desc(out.value, len(seqs), False)
+    return Desc(out.value, len(seqs), False, slot_kinds)
 
 
 def splice_workspace_bytes(desc: Desc) -> int:
@@ -211,6 +223,48 @@ def splice_plan_stats(desc: Desc, layer, step) -> dict:
     _check(lib().splice_plan_stats(desc.handle, layer, step, ctypes.byref(g), ctypes.byref(t),
                                    ctypes.byref(p), ctypes.byref(s)), "splice_plan_stats")
     return {"num_groups": g.value, "num_tiles": t.value, "prompt_visible": p.value, "suffix_visible": s.value}
+
+
+GROUP_DELTA = 0x100
+
+
+def splice_delta_bytes(desc: Desc) -> int:
+    return int(lib().splice_delta_bytes(desc.handle))
+
+
+def splice_delta_build(desc: Desc, k_clean, v_clean, k_donor, v_donor, delta, max_fraction=1.0, delta_bytes=None,
+                       stream=None) -> list:
+    """Encodes the stored donor spans into ``delta`` (a device buffer of
+    splice_delta_bytes bytes) and enters delta mode for the slots whose
+    encoded fraction is at most ``max_fraction``; returns every slot's
+    fraction (-1 for ZERO slots)."""
+    if delta_bytes is None:
+        delta_bytes = delta.numel() * delta.element_size()
+    n = len(_desc_slots(desc))
+    frac = (ctypes.c_float * n)()
+    _check(lib().splice_delta_build(desc.handle, _ptr(k_clean), _ptr(v_clean), _ptr(k_donor), _ptr(v_donor),
+                                    _ptr(delta), delta_bytes, float(max_fraction), frac, _stream(stream)),
+           "splice_delta_build")
+    return [float(f) for f in frac]
+
+
+def splice_delta_clear(desc: Desc, stream=None):
+    _check(lib().splice_delta_clear(desc.handle, _stream(stream)), "splice_delta_clear")
+
+
+def splice_debug_plan_delta(desc: Desc, slot_delta):
+    flags = (ctypes.c_uint8 * len(slot_delta))(*[1 if f else 0 for f in slot_delta])
+    _check(lib().splice_debug_plan_delta(desc.handle, flags), "splice_debug_plan_delta")
+
+
+def splice_debug_plan_rows(desc: Desc, layer, step) -> list:
+    """[(tile, group source, sequence, row mask)] of the prompt-span tiles at (layer, step)."""
+    n = _c_int()
+    _check(lib().splice_debug_plan_rows(desc.handle, layer, step, None, 0, ctypes.byref(n)), "splice_debug_plan_rows")
+    buf = (ctypes.c_int32 * (4 * max(1, n.value)))()
+    _check(lib().splice_debug_plan_rows(desc.handle, layer, step, buf, n.value, ctypes.byref(n)),
+           "splice_debug_plan_rows")
+    return [tuple(buf[4 * i:4 * i + 4]) for i in range(n.value)]
 
 
 def splice_debug_wait_timeout(desc: Desc, limit_us: int, stream=None):
