@@ -22,6 +22,8 @@ Legs (one JSON line on rank 0):
 * graph: each timed step's calls (every layer's append and attention)
   captured once into a CUDA graph before the timed region, then the K graphs
   replayed under the same events -- the fused-step launch mode;
+* delta: the same K steps in delta-donor mode (donor spans that share most
+  positions with the clean span encoded against it once, before timing);
 * cpu_baseline: the fp64 CPU oracle on a bounded sample of (sequence,
   layer, step) units of the same batch, on the host's cores.
 ``--impl reference`` times that oracle alone as the reference arm.
@@ -88,18 +90,37 @@ def read_peaks():
 # --------------------------------------------------------------------------
 # algorithmic bytes (what the method must move), from the source maps
 # --------------------------------------------------------------------------
-def algorithmic_bytes(sb, layer: int, step: int):
+def algorithmic_bytes(sb, layer: int, step: int, delta=None):
+    """Bytes per kernel kind at (layer, step).  ``delta`` = (slot flags,
+    encoded counts [prompts][stored slots][N][Hkv]) in delta mode: a reader
+    of an encoded slot reads its prompt's clean span (shared with the clean
+    readers) and the slot's encoded rows instead of the donor span."""
     from paper_2605_30574_gb300 import splice as S
     wl = sb.wl
     st = S.splice_plan_stats(sb.desc, layer, step)
     m = S.splice_debug_source_map(sb.desc, layer, step)
-    spans = {(sb.seqs[s].prompt, code) for s, code in enumerate(m) if code != S.SRC_ZERO}
+    kv_pos = wl.num_kv_heads * wl.head_dim * 4          # K + V bf16 of one position, all kv heads
+    spans, rows = set(), 0
+    for s, code in enumerate(m):
+        if code == S.SRC_ZERO:
+            continue
+        p = sb.seqs[s].prompt
+        if delta is not None and code >= S.SRC_DONOR0 and delta[0][code - S.SRC_DONOR0]:
+            spans.add((p, S.SRC_CLEAN))
+            spans.add((p, -int(code)))                  # the slot's encoded rows, counted below
+        else:
+            spans.add((p, code))
+    for p, code in spans:
+        if code < 0:
+            k = -code - S.SRC_DONOR0
+            stq = sum(1 for j in range(k) if wl.slot_kinds[j] != 0)
+            rows += int(delta[1][p - sb.p0, stq, layer].sum()) * wl.head_dim * 4
+    n_span = sum(1 for _, code in spans if code >= 0)
     n_read = sum(1 for code in m if code != S.SRC_ZERO)
-    kv_row = wl.num_kv_heads * wl.head_dim * 4          # K + V bf16 of one position, all kv heads
     q_bytes = wl.num_q_heads * wl.head_dim * 2
     return {
-        "prompt_span_pass": len(spans) * st["prompt_visible"] * kv_row + n_read * q_bytes,
-        "generated_span_pass": sb.B * st["suffix_visible"] * kv_row + sb.B * q_bytes,
+        "prompt_span_pass": n_span * st["prompt_visible"] * kv_pos + rows + n_read * q_bytes,
+        "generated_span_pass": sb.B * st["suffix_visible"] * kv_pos + sb.B * q_bytes,
         "merge": sb.B * wl.num_q_heads * wl.head_dim * 4,
         "append": sb.B * wl.num_kv_heads * wl.head_dim * 8 if step >= 1 else 0,
     }
@@ -393,6 +414,11 @@ def gpu_arm(args):
     if not args.no_graph:
         graph = graph_leg(sb, steps, qs, kn, vn, outs, run_step, world, dist)
 
+    # ---- delta: donor spans encoded against the clean spans ----
+    delta = None
+    if not args.no_delta and sb.Dst:
+        delta = delta_leg(sb, steps, qs, kn, vn, outs, run_step, world, dist, per_kind)
+
     # ---- e2e: host buffers through the C ABI, copies overlapped ----
     e2e = None
     if not args.no_e2e:
@@ -420,7 +446,7 @@ def gpu_arm(args):
                          "bytes_per_launch": per_kind[dom] // max(n_l, 1),
                          "ms_per_launch": ms_l / max(n_l, 1)},
             "kernels": kernels,
-            "e2e": e2e, "graph": graph, "gpu_launches": gpu_launches, "clocks": clk.summary(),
+            "e2e": e2e, "graph": graph, "delta": delta, "gpu_launches": gpu_launches, "clocks": clk.summary(),
             "cpu_baseline": cpu,
         }
         print(json.dumps(line))
@@ -462,6 +488,71 @@ def graph_leg(sb, steps, qs, kn, vn, outs, run_step, world, dist):
     return {"value": units / (ms / 1000.0), "unit": UNIT, "ms_per_step": ms / len(steps),
             "how": "each timed step (all layers: append + attention) captured once into a CUDA graph before "
                    "the timed region; the K graphs replayed under CUDA events"}
+
+
+def delta_leg(sb, steps, qs, kn, vn, outs, run_step, world, dist, plain_bytes, max_fraction=0.6):
+    """The K timed steps in delta-donor mode: the batch's stored donor spans
+    encoded against the clean spans once, before the timed region (slots
+    whose encoded fraction is at most max_fraction), then the same steps
+    timed under CUDA events; the prompt-span pass timed per launch after."""
+    import torch
+    from paper_2605_30574_gb300 import splice as S
+    wl, N = sb.wl, sb.wl.num_layers
+    buf = torch.empty(S.splice_delta_bytes(sb.desc), dtype=torch.uint8, device=sb.k_clean.device)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    frac = S.splice_delta_build(sb.desc, sb.k_clean, sb.v_clean, sb.k_donor, sb.v_donor, buf, max_fraction)
+    build_s = time.perf_counter() - t0
+    flags = [f >= 0 and f <= max_fraction for f in frac]
+    # encoded counts, from the buffer's count part
+    spans = sb.Pl * sb.Dst * N * wl.num_kv_heads
+    w32 = 4 * ((wl.prompt_len + 127) // 128)
+    count_off = (spans * w32 * 4 + 255) // 256 * 256
+    counts = buf[count_off: count_off + spans * 4].view(torch.int32).cpu().numpy().reshape(
+        sb.Pl, sb.Dst, N, wl.num_kv_heads)
+    for i, t in enumerate(steps[:2]):
+        run_step(t, qs[i], kn[i], vn[i], outs)
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    ev0.record()
+    for i, t in enumerate(steps):
+        run_step(t, qs[i], kn[i], vn[i], outs)
+    ev1.record()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    ms = ev0.elapsed_time(ev1)
+    S.splice_check_device_error(sb.desc)
+    per_kind = {"append": 0, "prompt_span_pass": 0, "generated_span_pass": 0, "merge": 0}
+    for t in steps:
+        for l in range(N):
+            for k, v in algorithmic_bytes(sb, l, t, (flags, counts)).items():
+                per_kind[k] += v
+    S.splice_profile_enable(sb.desc, True)
+    S.splice_profile_read(sb.desc)
+    for i, t in enumerate(steps):
+        run_step(t, qs[i], kn[i], vn[i], outs)
+    torch.cuda.synchronize()
+    prof = S.splice_profile_read(sb.desc)
+    S.splice_profile_enable(sb.desc, False)
+    S.splice_delta_clear(sb.desc)
+    del buf
+    units = sb.B * len(steps)
+    ms, units = reduce_timing(ms, units, dist if world > 1 else None, torch.device("cuda", torch.cuda.current_device()))
+    pp = prof["prompt_span_pass"]
+    return {"value": units / (ms / 1000.0), "unit": UNIT, "ms_per_step": ms / len(steps),
+            "slot_fraction": [round(f, 4) for f in frac], "slots_encoded": [int(f) for f in flags],
+            "encode_s": round(build_s, 3),
+            "prompt_span_algorithmic_GB_per_step": round(per_kind["prompt_span_pass"] / len(steps) / 1e9, 3),
+            "prompt_span_algorithmic_GB_per_step_plain": round(plain_bytes["prompt_span_pass"] / len(steps) / 1e9, 3),
+            "prompt_span_pass_ms_per_step": round(pp[1] / len(steps), 3),
+            "prompt_span_pass_GBps": round(per_kind["prompt_span_pass"] / (pp[1] / 1000.0) / 1e9, 1) if pp[1] else None,
+            "how": f"stored donor slots with at most {max_fraction:.0%} of their positions differing from the clean "
+                   "span encoded once before the timed region (splice_delta_build); readers of an encoded slot "
+                   "read the clean span with those positions masked plus the encoded rows; same K steps"}
 
 
 def e2e_leg(sb, steps, qs, kn, vn, run_step, dev):
@@ -535,6 +626,7 @@ def main(argv=None):
     ap.add_argument("--batch", type=int, default=0)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-graph", action="store_true")
+    ap.add_argument("--no-delta", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args(argv)
     if args.impl == "reference":
