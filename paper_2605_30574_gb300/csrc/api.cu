@@ -487,7 +487,11 @@ splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const spl
     // kMaxPrefixSplits prompt-span partial slots.
     const int max_splits = d->delta_on ? splice::kMaxPrefixSplits / 2 : splice::kMaxPrefixSplits;
     int tc_split = 0, tc_keys = 0;
-    if (p_vis > 0) tc_keys = splice::prefix_tc_split_keys(sh.head_dim, p_vis, max_splits, &tc_split);
+    int bounds[splice::kMaxPrefixSplits + 1] = {0};
+    if (p_vis > 0) {
+        tc_split = splice::prefix_tc_splits(sh.head_dim, p_vis, max_splits, bounds);
+        tc_keys = bounds[1];           // the longest split
+    }
     p.nsp = tc_split;
     p.n_span_tiles = d->plan.table_span_tiles[tab];
     p.group_mask = d->d_group_mask;
@@ -550,7 +554,7 @@ splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const spl
         }
         const bool overlap = gs_launched && !d->profiling;
         e = timed_launch(d, 1, stream, [&] {
-            return splice::launch_prefix_tc(p, d->maps, tc_keys, stream, overlap);
+            return splice::launch_prefix_tc(p, d->maps, bounds, tc_keys, stream, overlap);
         });
         if (e != cudaSuccess) return cuda_fail(e, "prompt-span tensor-core pass launch");
     }

@@ -148,15 +148,18 @@ struct Bars {
 
 struct TcParams {
     AttnParams a;
-    int split_keys;     // keys per split (multiple of BN)
-    int n_span_items;   // items [0, n_span_items) read stored spans, the rest delta rows
+    int sb[kMaxPrefixSplits + 1];   // split boundaries of a stored span, relative to p_lo (multiples of BN)
+    int delta_keys;                 // keys per split of the delta rows (multiple of BN)
+    int n_span_items;               // items [0, n_span_items) read stored spans, the rest delta rows
     int n_items;
 };
 
 // Work item -> tile, kv head, split (consecutive items = consecutive tiles
 // of one (head, split), so a group's tiles read its span at about the same
-// time and share it in L2).  Items over stored spans come first, then the
-// items over delta rows (their own split count).
+// time and share it in L2; split-major, so the run-time queue hands out the
+// first -- longest -- split of every span before the shorter ones and the
+// launch ends on short items).  Items over stored spans come first, then
+// the items over delta rows (their own split count).
 struct ItemInfo {
     int h, split, first, nseq, k0, k1, nblk, prompt;
     int store;          // 0 clean, 1 donor, 2 delta rows
@@ -171,16 +174,16 @@ __device__ __forceinline__ ItemInfo item_info(const AttnParams& P, const TcParam
     if (item < tp.n_span_items) {
         tile = item % P.n_span_tiles;
         const int hs = item / P.n_span_tiles;
-        split = hs % P.nsp;
-        it.h = hs / P.nsp;
+        it.h = hs % P.Hkv;
+        split = hs / P.Hkv;
         it.split = split;                      // partial slot
     } else {
         const int nd = P.n_tiles - P.n_span_tiles;
         const int j = item - tp.n_span_items;
         tile = P.n_span_tiles + j % nd;
         const int hs = j / nd;
-        split = hs % P.nsd;
-        it.h = hs / P.nsd;
+        it.h = hs % P.Hkv;
+        split = hs / P.Hkv;
         it.split = P.nsp + split;              // after the span's own partials
     }
     const int4 tl = reinterpret_cast<const int4*>(P.tiles)[tile];
@@ -194,8 +197,8 @@ __device__ __forceinline__ ItemInfo item_info(const AttnParams& P, const TcParam
         span = ((long(it.prompt) * P.Dst + st) * P.N + P.layer) * P.Hkv + it.h;
         it.store = 2;
         it.masked = false;
-        it.k0 = split * tp.split_keys;
-        it.k1 = min(P.dcount[span], it.k0 + tp.split_keys);
+        it.k0 = split * tp.delta_keys;
+        it.k1 = min(P.dcount[span], it.k0 + tp.delta_keys);
     } else {
         if (code == int(SPLICE_SRC_CLEAN)) {
             span = (long(it.prompt) * P.N + P.layer) * P.Hkv + it.h;
@@ -207,8 +210,8 @@ __device__ __forceinline__ ItemInfo item_info(const AttnParams& P, const TcParam
             it.store = 1;
             it.masked = false;
         }
-        it.k0 = P.p_lo + split * tp.split_keys;
-        it.k1 = min(P.p_hi, it.k0 + tp.split_keys);
+        it.k0 = P.p_lo + tp.sb[split];
+        it.k1 = P.p_lo + tp.sb[split + 1];
     }
     it.span_row = span * P.Tp;
     it.nblk = it.k1 > it.k0 ? (it.k1 - it.k0 + Cfg<D>::BN - 1) / Cfg<D>::BN : 0;
@@ -900,24 +903,46 @@ int prefix_tc_box_rows(int d) {
     return d == 64 ? Cfg<64>::BN : (d == 128 ? Cfg<128>::BN : Cfg<256>::BN);
 }
 
-int prefix_tc_split_keys(int d, int p_vis, int max_splits, int* nsplit) {
-    const int bn = prefix_tc_box_rows(d);
+int prefix_tc_splits(int d, int p_vis, int max_splits, int* bounds) {
     // Splits depend only on the visible span length (and the cap), so a
     // row's arithmetic never depends on which other rows share its tile or
-    // launch.
-    int ns = (p_vis + 1023) / 1024;
-    ns = ns < 1 ? 1 : (ns > max_splits ? max_splits : ns);
-    int keys = (p_vis + ns - 1) / ns;
-    keys = (keys + bn - 1) / bn * bn;
-    ns = (p_vis + keys - 1) / keys;
-    *nsplit = ns;
-    return keys;
+    // launch.  Every item gathers its tile's queries and stores its partial
+    // states, so fewer, longer items move fewer bytes: splits of kSplitKeys
+    // keys, all but the last full.  A longer span ends in a shorter split,
+    // which the split-major item order hands out last, so a launch ends on
+    // short items.  Past the cap, the blocks are shared out evenly.
+    constexpr int kSplitKeys = 3072;
+    const int bn = prefix_tc_box_rows(d);
+    const int nb = (p_vis + bn - 1) / bn;
+    const int full = kSplitKeys / bn;
+    int ns = (nb + full - 1) / full;
+    bounds[0] = 0;
+    if (ns <= max_splits) {
+        for (int i = 0; i < ns; ++i) {
+            const int b = bounds[i] + full * bn;
+            bounds[i + 1] = b < p_vis ? b : p_vis;
+        }
+        return ns;
+    }
+    ns = max_splits;
+    for (int i = 0; i < ns; ++i) {
+        const int blocks = nb / ns + (i < nb % ns ? 1 : 0);
+        const int b = bounds[i] + blocks * bn;
+        bounds[i + 1] = b < p_vis ? b : p_vis;
+    }
+    return ns;
 }
 
-int launch_prefix_tc(const AttnParams& p, const void* maps, int split_keys, void* stream, bool overlap_previous) {
+int launch_prefix_tc(const AttnParams& p, const void* maps, const int* bounds, int delta_keys, void* stream,
+                     bool overlap_previous) {
     const CUtensorMap* m = static_cast<const CUtensorMap*>(maps);
     const int n_span_items = p.n_span_tiles * p.Hkv * p.nsp;
-    TcParams tp{p, split_keys, n_span_items, n_span_items + (p.n_tiles - p.n_span_tiles) * p.Hkv * p.nsd};
+    TcParams tp{};
+    tp.a = p;
+    for (int i = 0; i <= p.nsp && i <= kMaxPrefixSplits; ++i) tp.sb[i] = bounds[i];
+    tp.delta_keys = delta_keys;
+    tp.n_span_items = n_span_items;
+    tp.n_items = n_span_items + (p.n_tiles - p.n_span_tiles) * p.Hkv * p.nsd;
     if (tp.n_items <= 0) return 0;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     int r = int(cudaErrorInvalidValue);

@@ -131,14 +131,18 @@ int launch_wait_timeout(unsigned* err, unsigned long long limit_ns, void* stream
 // Tensor-core prompt-span pass.  A tensor map is a 128-byte CUtensorMap.
 int make_kv_tensor_map(void* out_map, const void* base, long rows, int d, int box_rows);
 int prefix_tc_box_rows(int d);
-// Keys per split of a visible span of p_vis keys and the number of splits
-// (at most max_splits).
-int prefix_tc_split_keys(int d, int p_vis, int max_splits, int* nsplit);
+// Key splits of a visible span of p_vis keys: returns their number n (at
+// most max_splits) and writes bounds[0 .. n], 0 = bounds[0] < ... <
+// bounds[n] = p_vis, every inner bound a multiple of the key block.
+int prefix_tc_splits(int d, int p_vis, int max_splits, int* bounds);
 // maps: six tensor maps -- clean K, V; donor K, V; delta rows K, V.
-// overlap_previous: the launch directly follows the generated-span pass on
-// the same stream and may start while that pass finishes (programmatic
-// dependent launch); the kernel waits for it before it exits.
-int launch_prefix_tc(const AttnParams& p, const void* maps, int split_keys, void* stream, bool overlap_previous);
+// bounds: the span splits (p.nsp + 1 values); delta_keys: keys per split of
+// the delta rows.  overlap_previous: the launch directly follows the
+// generated-span pass on the same stream and may start while that pass
+// finishes (programmatic dependent launch); the kernel waits for it before
+// it exits.
+int launch_prefix_tc(const AttnParams& p, const void* maps, const int* bounds, int delta_keys, void* stream,
+                     bool overlap_previous);
 
 // Delta encoding of every stored donor span (one CTA per span): bits of the
 // positions whose K or V row differs from the clean span, their count, and

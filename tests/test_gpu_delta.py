@@ -115,6 +115,8 @@ EDGE = [
     ("g2_d256", 3, 4, 2, 256, 2, 200, (WL.BLANK, WL.ZERO, WL.DIFF_ALGO), 12),
     ("g8_d128", 2, 16, 2, 128, 1, 129, (WL.DIFF_ALGO, WL.ZERO), 6),
     ("g3_d64_long", 2, 6, 2, 64, 1, 1100, (WL.SAME_ALGO, WL.BLANK), 300),
+    # delta mode caps the span at four splits: 13000 keys are shared out evenly
+    ("long_span_4_splits", 1, 4, 2, 64, 1, 13000, (WL.SAME_ALGO, WL.ZERO), 3),
 ]
 
 

@@ -134,6 +134,8 @@ EDGE = [
     ("g8_d128", 2, 16, 2, 128, 1, 129, (WL.DIFF_ALGO, WL.ZERO), 6, 0, 0),
     ("g3_d64_long", 2, 6, 2, 64, 1, 1100, (WL.BLANK,), 700, 0, 0),
     ("window_below_suffix", 3, 8, 2, 64, 1, 64, (WL.ZERO, WL.BLANK), 50, 20, 0),
+    # five prompt-span splits: four of 3072 keys and a short last one
+    ("long_span_5_splits", 1, 4, 2, 64, 1, 13000, (WL.SAME_ALGO, WL.ZERO), 3, 0, 0),
 ]
 
 
