@@ -507,12 +507,15 @@ splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const spl
     }
     {
         // Generated-span items: (sequence, kv head, row chunk, key split).
-        // Split so every resident warp gets about four items, but keep at
-        // least 64 keys per split.
+        // Split so every resident warp gets about two items, but keep at
+        // least 64 keys per split.  Every split costs a partial state to
+        // write and merge; the prompt-span pass queued behind this one fills
+        // the SMs its last warps leave idle, so few splits pay off even
+        // where the items do not share out evenly over the warps.
         const int G = sh.num_q_heads / sh.num_kv_heads;
         const int gt = G % 4 == 0 ? 4 : (G % 2 == 0 ? 2 : 1);
         const long base_items = long(d->B) * sh.num_kv_heads * (G / gt);
-        const long want = 4L * splice::generated_span_resident_warps(sh.head_dim);
+        const long want = 2L * splice::generated_span_resident_warps(sh.head_dim);
         int ns = int(std::min<long>(splice::kMaxSuffixSplits, std::max<long>(1, (want + base_items - 1) / base_items)));
         ns = std::min(ns, std::max(1, s_vis / 64));
         p.nss = s_vis > 0 ? ns : 0;

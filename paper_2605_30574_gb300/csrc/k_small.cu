@@ -32,9 +32,11 @@ __global__ void append_kernel(const uint4* __restrict__ kn, const uint4* __restr
 
 // One warp per output row: the partial states of the prompt-span and the
 // generated-span passes (and the ZERO closed form) -> out.  Rows with up to
-// eight live partials take the one-round-trip path.
+// four partials -- the common case -- take the one-round-trip path, whose
+// few registers let six blocks (48 warps) share an SM, so more rows' loads
+// are in flight at once.
 template <int D>
-__global__ void __launch_bounds__(256, 4) merge_kernel(AttnParams P) {
+__global__ void __launch_bounds__(256, 6) merge_kernel(AttnParams P) {
     // Launched behind the prompt-span pass as a programmatic dependent, this
     // grid may start before that pass has finished: wait for it (and so for
     // the generated-span pass it waited for) before reading any partial.
@@ -43,7 +45,7 @@ __global__ void __launch_bounds__(256, 4) merge_kernel(AttnParams P) {
     const long warp = (long(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
     if (warp >= long(P.B) * P.Hq) return;
-    if (!merge_row_fast<D, 8>(P, warp, lane)) merge_row(P, warp, lane);
+    if (!merge_row_fast<D, 4>(P, warp, lane)) merge_row(P, warp, lane);
 }
 
 }  // namespace
