@@ -51,6 +51,9 @@ struct splice_desc {
     std::vector<uint8_t> slot_delta;    // [Dslots]
     bool delta_on = false;
     char* delta = nullptr;
+    // (layer, step) of the append launched last, if it was the last launch
+    // through this descriptor (-1 otherwise)
+    int append_layer = -1, append_step = -1;
     int delta_max = 0;
     // TMA tensor maps of the clean and donor stores and of the delta rows
     // (K, V each), rebuilt when the store pointers change.
@@ -409,11 +412,14 @@ splice_status suffix_kv_append(splice_desc* d, int layer, int step, const splice
     if (g.err != cudaSuccess) return cuda_fail(g.err, "cudaSetDevice");
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "earlier CUDA error");
+    d->append_layer = d->append_step = -1;
     e = timed_launch(d, 0, stream, [&] {
         return splice::launch_append(k_new, v_new, k_suffix, v_suffix, d->B, d->shape.num_layers,
                                      d->shape.num_kv_heads, d->shape.head_dim, d->T, layer, step, stream);
     });
     if (e != cudaSuccess) return cuda_fail(e, "append launch");
+    d->append_layer = layer;
+    d->append_step = step;
     return SPLICE_OK;
 }
 
@@ -443,6 +449,11 @@ splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const spl
     const splice_model_shape& sh = d->shape;
     const int tab = d->plan.table_of(layer, step);
     const splice::Visible vis = splice::visible_keys(sh, d->Tp, layer, step);
+    // The generated-span pass may read its older entries while the append
+    // launched right before it still runs, if that append wrote this layer
+    // and step (its only write is the entry this call reads last).
+    const bool dep_late = d->append_layer == layer && d->append_step == step && !d->profiling;
+    d->append_layer = d->append_step = -1;
     const size_t rows = size_t(d->B) * sh.num_q_heads;
     AttnParams p{};
     p.q = q;
@@ -497,6 +508,7 @@ splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const spl
     p.group_mask = d->d_group_mask;
     p.slot_delta = d->d_slot_delta;
     p.delta_on = d->delta_on ? 1 : 0;
+    p.dep_late = dep_late ? 1 : 0;
     p.nsd = 0;
     if (d->delta_on) {
         const DeltaLayout dl = delta_layout(d);
@@ -591,6 +603,7 @@ splice_status splice_delta_build(splice_desc* d, const splice_bf16* k_clean, con
     if (e != cudaSuccess) return cuda_fail(e, "earlier CUDA error");
     const splice_model_shape& sh = d->shape;
     char* b = static_cast<char*>(delta);
+    d->append_layer = d->append_step = -1;
     e = cudaError_t(splice::launch_delta_build(
         k_clean, v_clean, k_donor, v_donor, reinterpret_cast<uint32_t*>(b + dl.mask_off),
         reinterpret_cast<int32_t*>(b + dl.count_off), reinterpret_cast<uint16_t*>(b + dl.k_off),
@@ -748,6 +761,7 @@ splice_status splice_debug_wait_timeout(splice_desc* d, unsigned limit_us, void*
     if (limit_us == 0 || limit_us > 1000000u) return fail(SPLICE_EINVAL, "limit_us %u not in [1, 1000000]", limit_us);
     DeviceGuard g(d->device);
     if (g.err != cudaSuccess) return cuda_fail(g.err, "cudaSetDevice");
+    d->append_layer = d->append_step = -1;
     cudaError_t e = cudaError_t(splice::launch_wait_timeout(d->d_err, 1000ull * limit_us, stream));
     if (e != cudaSuccess) return cuda_fail(e, "wait-timeout launch");
     return SPLICE_OK;

@@ -116,12 +116,20 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
     extern __shared__ __align__(128) uint8_t smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     // Launched as a programmatic dependent of whatever precedes it on the
-    // stream (usually the append of this step's K/V): wait for that grid to
-    // complete before reading anything.  A no-op for a plain launch.
-    asm volatile("griddepcontrol.wait;" ::: "memory");
-    // The prompt-span pass queued behind this grid reads nothing it writes:
-    // let it start as soon as SMs free up.
+    // stream, this grid may start before that grid has finished.  Where the
+    // host knows the preceding grid is the append of this very layer and
+    // step (P.dep_late), which writes generated-span entry step - 1 and
+    // nothing else this pass reads, the wait for it comes only before the
+    // first copy of a block that holds that entry, and the blocks before it
+    // stream in the meantime; otherwise it comes first.  A no-op for a plain
+    // launch.  The prompt-span pass queued behind this grid reads nothing it
+    // writes: let it start as soon as SMs free up.
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    bool dep_done = false;
+    if (!P.dep_late) {
+        asm volatile("griddepcontrol.wait;" ::: "memory");
+        dep_done = true;
+    }
     uint8_t* ws = smem + warp * C::PER_WARP;
     const uint32_t wbase = tc::smem_u32(ws);
     const uint32_t bar0 = wbase + C::OFF_BAR;
@@ -157,6 +165,10 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
         const int j = iss.k0 + iss_b * 16;
         const int nk = min(16, iss.k1 - j);
         const uint32_t bytes = uint32_t(nk) * C::ROW;
+        if (!dep_done && j + nk >= P.s_hi) {
+            asm volatile("griddepcontrol.wait;" ::: "memory");
+            dep_done = true;
+        }
         if (lane == 0) {
             const uint32_t dst = wbase + stg * C::STAGE;
             tc::mbar_arrive_expect_tx(bar0 + 8 * stg, 2 * bytes);
@@ -362,6 +374,9 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
             }
         }
     }
+    // This grid's completion implies the preceding grid's for whatever is
+    // queued after it.
+    if (!dep_done) asm volatile("griddepcontrol.wait;" ::: "memory");
     // Copies still in flight (only after an abort) must land before exit.
     for (; consumed < issued; ++consumed) {
         volatile int no_abort = 0;

@@ -105,6 +105,7 @@ struct AttnParams {
     int nsp, nss;                 // splits of the prompt span / generated span
     int nsd;                      // splits of the delta rows (delta mode)
     int delta_on, delta_w32;
+    int dep_late;                 // the preceding grid is this layer and step's append (see gs_kernel)
     int p_chunk, s_chunk;         // keys per split
     int n_tiles;
     int n_span_tiles;             // tiles [0, n_span_tiles) read stored spans, the rest delta rows

@@ -203,3 +203,44 @@ def test_two_descriptors_interleaved_on_one_stream():
         assert torch.equal(b.out, alone_b[(l, t)]), ("b", l, t)
     S.splice_check_device_error(a.desc)
     S.splice_check_device_error(b.desc)
+
+
+def test_attention_reads_the_entry_appended_right_before():
+    """The generated-span pass may stream its older entries while the
+    append launched right before it (same layer and step) still runs; the
+    entry that append writes must still be read only after it lands.  The
+    slot is poisoned with large values first, so reading it early would
+    swamp the softmax.  Also an append of an older slot followed by an
+    attention call at a later step: the pass then waits for the append
+    before it reads anything."""
+    from test_gpu_parity import oracle_rows
+    from parity_util import CachedInputs
+    wl = WL.get("qwen3-8b-ladder")
+    wl = WL.Workload("late-wait", 3, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, 2, 256, wl.slot_kinds, 64,
+                     (0, 1, 3), (0, 16), wl.scaffold_head, wl.scaffold_tail, batch=10 ** 6)
+    sb = SweepBatch(wl, seqs=wl.sequences())
+    inp = CachedInputs(wl)
+    poison = torch.tensor(40.0, dtype=torch.bfloat16)
+    for l, t in ((0, 1), (1, 17), (2, 64), (1, 33)):
+        sb.gen_inputs(l, t)
+        torch.cuda.synchronize()
+        sb.k_suffix[:, l, :, t - 1] = poison.cuda()
+        sb.v_suffix[:, l, :, t - 1] = poison.cuda()
+        sb.append(l, t)
+        sb.attn(l, t)
+        out = sb.out.cpu().numpy()
+        ref = oracle_rows(wl, inp, sb.seqs, l, t, range(sb.B))
+        assert_close(out, ref, f"late wait l={l} t={t}")
+    # re-append an older slot, then attend a later step of the same layer
+    l, t_old, t = 1, 10, 30
+    sb.gen_inputs(l, t_old)
+    torch.cuda.synchronize()
+    sb.k_suffix[:, l, :, t_old - 1] = poison.cuda()
+    sb.v_suffix[:, l, :, t_old - 1] = poison.cuda()
+    sb.append(l, t_old)
+    sb.gen_inputs(l, t)
+    sb.attn(l, t)
+    out = sb.out.cpu().numpy()
+    ref = oracle_rows(wl, inp, sb.seqs, l, t, range(sb.B))
+    assert_close(out, ref, f"older slot l={l} t={t}")
+    S.splice_check_device_error(sb.desc)
