@@ -62,3 +62,51 @@ def test_decode_step_graph_replays_bit_exact(step):
     from paper_2605_30574_gb300 import splice as S
     S.splice_check_device_error(sb.desc)
     sb.close()
+
+
+def test_decode_step_graph_in_delta_mode():
+    """Delta-donor mode captures and replays like the default mode: the
+    replayed step equals the same calls issued one by one, replay after
+    replay, and both are within the path's tolerance of the fp64 oracle on
+    sampled rows (the oracle reads the donor spans themselves)."""
+    import numpy as np
+    import oracle
+    from parity_util import CachedInputs, assert_close
+    from paper_2605_30574_gb300 import splice as S
+    wl = ladder_slice(layers=4)
+    sb = SweepBatch(wl, 0)
+    buf = torch.empty(S.splice_delta_bytes(sb.desc), dtype=torch.uint8, device="cuda")
+    frac = S.splice_delta_build(sb.desc, sb.k_clean, sb.v_clean, sb.k_donor, sb.v_donor, buf, 0.6)
+    assert sum(1 for f in frac if 0 <= f <= 0.6) == 2        # SAME_ALGO and DIFF_ALGO
+    step, N = 300, wl.num_layers
+    qs, kns, vns = [], [], []
+    for l in range(N):
+        sb.gen_inputs(l, step)
+        qs.append(sb.q.clone())
+        kns.append(sb.k_new.clone())
+        vns.append(sb.v_new.clone())
+    outs_eager = [torch.empty_like(sb.out) for _ in range(N)]
+    for l in range(N):
+        sb.append(l, step, kns[l], vns[l])
+        sb.attn(l, step, q=qs[l], out=outs_eager[l])
+    torch.cuda.synchronize()
+    outs_graph = [torch.full_like(sb.out, float("nan")) for _ in range(N)]
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for l in range(N):
+            sb.append(l, step, kns[l], vns[l])
+            sb.attn(l, step, q=qs[l], out=outs_graph[l])
+    for _ in range(2):
+        for o in outs_graph:
+            o.fill_(float("nan"))
+        g.replay()
+        torch.cuda.synchronize()
+        for l in range(N):
+            assert torch.equal(outs_graph[l], outs_eager[l]), f"layer {l}"
+    inp = CachedInputs(wl)
+    rows = list(range(0, sb.B, 7))
+    for l in (0, N - 1):
+        ref = np.stack([oracle.decode_attn(wl, inp, s, sb.seqs[s], l, step) for s in rows])
+        assert_close(outs_graph[l][torch.tensor(rows, device="cuda")].cpu().numpy(), ref, f"delta graph l={l}")
+    S.splice_check_device_error(sb.desc)
+    sb.close()

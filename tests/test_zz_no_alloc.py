@@ -73,3 +73,26 @@ def test_static_scratch_refuses_oversized_descriptor():
     assert e.value.status == S.EINVAL
     assert "static maximum" in str(e.value)
     d.close()
+
+
+def test_static_scratch_in_delta_mode():
+    """The no-allocation entry point runs delta-donor mode like the
+    workspace entry point (the delta buffer is the caller's, allocated once
+    at setup)."""
+    base = WL.get("qwen3-8b-ladder")
+    wl = WL.Workload("ladder-slice-delta", 4, base.num_q_heads, base.num_kv_heads, base.head_dim, 2, 1024,
+                     base.slot_kinds, 400, (0, 2, 4), base.W_values, base.scaffold_head, base.scaffold_tail,
+                     batch=100)
+    sb = SweepBatch(wl, 0)
+    buf = torch.empty(S.splice_delta_bytes(sb.desc), dtype=torch.uint8, device="cuda")
+    S.splice_delta_build(sb.desc, sb.k_clean, sb.v_clean, sb.k_donor, sb.v_donor, buf, 0.6)
+    for layer, step in ((1, 20), (3, 300)):
+        sb.gen_inputs(layer, step)
+        sb.append(layer, step)
+        sb.attn(layer, step)
+        want = sb.out.clone()
+        got = torch.full_like(sb.out, float("nan"))
+        _static_call(sb, layer, step, got)
+        torch.cuda.synchronize()
+        assert torch.equal(got, want), (layer, step)
+    S.splice_check_device_error(sb.desc)
