@@ -12,8 +12,11 @@
 //     -- is in flight while the current one is computed;
 //   * a key row of d values is split over LPK = d / 16 lanes (16 dims each,
 //     two 16-byte chunks); q . k partial sums are reduced across the LPK
-//     lanes through a small shared-memory transpose (each lane ends with a
-//     few full logits), then probabilities are shared back the same way;
+//     lanes through a small shared-memory transpose (lane dl of a key group
+//     ends with the full logits v = dl, dl + LPK, ..., all of query row
+//     dl mod GT, read bank-conflict free), then probabilities are shared
+//     back the same way; each lane sums the probabilities of its own
+//     logits and the row sums are reduced once per item;
 //   * packed fp32x2 FMAs (FFMA2) for both q . k and p . v;
 //   * online softmax with a lazily moved reference max: the common path
 //     needs no rescale and no cross-lane max.
@@ -71,15 +74,21 @@ struct GS {
     static constexpr int VPL = NV >= LPK ? NV / LPK : 1;   // logits reduced by each lane
     static constexpr int WARPS = D == 256 ? 2 : 4;
     static constexpr int RED = NV + 4;              // padded floats per lane in the reduce buffer
+    // floats per key group in the reduce buffer: a multiple of 32 plus LPK,
+    // so the LPK partials of logit v of the KPW groups land in 32 distinct banks
+    static constexpr int GSTRIDE = (LPK * RED + 31) / 32 * 32 + LPK;
+    static constexpr int VPL_LIVE = NV >= LPK ? LPK : NV;   // lanes of a group holding distinct logits
     static constexpr uint32_t ROW = D * 2;          // bytes of one key row
     static constexpr uint32_t STAGE = BK * ROW * 2; // K + V block
     // per-warp shared memory: 2 stages, reduce buffer, probability pairs, 2 barriers
     static constexpr uint32_t OFF_RED = 2 * STAGE;
-    static constexpr uint32_t OFF_PP = OFF_RED + 32 * RED * 4;
+    static constexpr uint32_t OFF_PP = OFF_RED + KPW * GSTRIDE * 4;
     static constexpr uint32_t OFF_BAR = OFF_PP + KPW * NV * 8;
     static constexpr uint32_t PER_WARP = (OFF_BAR + 16 + 127) / 128 * 128;
     static constexpr uint32_t SMEM = WARPS * PER_WARP;
     static_assert(NV % 4 == 0 || NV < 4, "reduce layout");
+    static_assert(NV < LPK || NV == VPL * LPK, "every logit of a group owned by one lane");
+    static_assert(LPK % GT == 0, "the logits of a lane belong to one query row");
 };
 
 // Where the keys of one work item live.
@@ -137,6 +146,7 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
     float2* pp = reinterpret_cast<float2*>(ws + C::OFF_PP);
 
     const int gi = lane / C::LPK, dl = lane % C::LPK;
+    const int g_mine = dl % GT;
     const int c0 = dl, c1 = dl + C::LPK;
     const int gwarp = blockIdx.x * C::WARPS + warp;
     const int nwarps = gridDim.x * C::WARPS;
@@ -205,15 +215,18 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
                 q2[g][i] = make_float2(f.x * P.scale_log2, f.y * P.scale_log2);
             }
         }
-        float m[GT], l[GT];
+        // m: every row's reference max (the same in every lane of a key
+        // group); m_mine: that of row g_mine, the row of this lane's logits;
+        // l_mine: this lane's share of row g_mine's sum
+        float m[GT];
         float2 o2[GT][8];
 #pragma unroll
         for (int g = 0; g < GT; ++g) {
             m[g] = -INFINITY;
-            l[g] = 0.f;
 #pragma unroll
             for (int i = 0; i < 8; ++i) o2[g][i] = make_float2(0.f, 0.f);
         }
+        float m_mine = -INFINITY, l_mine = 0.f;
 
         for (int b = 0; b < it.nblk; ++b) {
             const int stg = consumed & 1;
@@ -246,7 +259,8 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
                 }
             }
             // ---- transpose-reduce across the LPK lanes of the group ----
-            float* myred = red + lane * C::RED;
+            float* gred = red + gi * C::GSTRIDE;
+            float* myred = gred + dl * C::RED;
             if constexpr (C::NV % 4 == 0) {
 #pragma unroll
                 for (int v = 0; v < C::NV; v += 4)
@@ -257,50 +271,57 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
             }
             __syncwarp();
             float sv[C::VPL];
-            int gv[C::VPL];
             bool need = false;
 #pragma unroll
             for (int i = 0; i < C::VPL; ++i) {
-                const int v = (dl * C::VPL + i) % C::NV;
-                float acc = 0.f;
+                const int v = (dl + C::LPK * i) % C::NV;
+                float part[C::LPK];
 #pragma unroll
-                for (int q = 0; q < C::LPK; ++q) acc += red[(gi * C::LPK + q) * C::RED + v];
+                for (int q = 0; q < C::LPK; ++q) part[q] = gred[q * C::RED + v];
+#pragma unroll
+                for (int w = C::LPK / 2; w > 0; w >>= 1) {
+#pragma unroll
+                    for (int q = 0; q < w; ++q) part[q] += part[q + w];
+                }
                 const int u = v / GT;
-                gv[i] = v % GT;
                 const bool valid = jb + u * C::KPW + gi < it.k1;
-                sv[i] = valid ? acc : -INFINITY;
-                need |= sv[i] > m[gv[i]] + kTau;
+                sv[i] = valid ? part[0] : -INFINITY;
+                need |= sv[i] > m_mine + kTau;
             }
             if (__any_sync(kFull, need)) {
                 // rare: some row's reference max moves; share every logit of
                 // the group and recompute the per-row block maxima
                 __syncwarp();
 #pragma unroll
-                for (int i = 0; i < C::VPL; ++i) red[(gi * C::LPK) * C::RED + (dl * C::VPL + i) % C::NV] = sv[i];
+                for (int i = 0; i < C::VPL; ++i) gred[(dl + C::LPK * i) % C::NV] = sv[i];
                 __syncwarp();
 #pragma unroll
                 for (int g = 0; g < GT; ++g) {
                     float mb = -INFINITY;
 #pragma unroll
-                    for (int u = 0; u < C::U; ++u) mb = fmaxf(mb, red[(gi * C::LPK) * C::RED + u * GT + g]);
+                    for (int u = 0; u < C::U; ++u) mb = fmaxf(mb, gred[u * GT + g]);
                     if (mb > m[g] + kTau) {
                         const float alpha = ex2(m[g] - mb);
-                        l[g] *= alpha;
+                        if (g == g_mine) l_mine *= alpha;
                         const float2 a2 = make_float2(alpha, alpha);
 #pragma unroll
                         for (int i = 0; i < 8; ++i) o2[g][i] = __fmul2_rn(o2[g][i], a2);
                         m[g] = mb;
                     }
                 }
+#pragma unroll
+                for (int g = 0; g < GT; ++g)
+                    if (g == g_mine) m_mine = m[g];
             }
             // ---- probabilities, shared back as (p, p) pairs ----
             __syncwarp();
             float2* mypp = pp + gi * C::NV;
+            const float mg = m_mine == -INFINITY ? 0.f : m_mine;
 #pragma unroll
             for (int i = 0; i < C::VPL; ++i) {
-                const float mg = m[gv[i]] == -INFINITY ? 0.f : m[gv[i]];
                 const float p = ex2(sv[i] - mg);
-                if (C::NV >= C::LPK || dl < C::NV) mypp[(dl * C::VPL + i) % C::NV] = make_float2(p, p);
+                l_mine += p;
+                if (C::NV >= C::LPK || dl < C::NV) mypp[(dl + C::LPK * i) % C::NV] = make_float2(p, p);
             }
             __syncwarp();
             float2 p2[C::NV];
@@ -309,11 +330,6 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
                 const float4 t = *reinterpret_cast<const float4*>(mypp + v);
                 p2[v] = make_float2(t.x, t.y);
                 if (v + 1 < C::NV) p2[v + 1] = make_float2(t.z, t.w);
-            }
-#pragma unroll
-            for (int u = 0; u < C::U; ++u) {
-#pragma unroll
-                for (int g = 0; g < GT; ++g) l[g] += p2[u * GT + g].x;
             }
             // ---- o += p . v over this lane's 16 dims ----
 #pragma unroll
@@ -338,6 +354,16 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
             issue_next();
         }
         if (!ok) break;
+
+        // ---- row sums of the group: the lanes holding distinct logits ----
+        float l[GT];
+#pragma unroll
+        for (int g = 0; g < GT; ++g) {
+            float x = (g == g_mine && dl < C::VPL_LIVE) ? l_mine : 0.f;
+#pragma unroll
+            for (int off = 1; off < C::LPK; off <<= 1) x += __shfl_xor_sync(kFull, x, off);
+            l[g] = x;
+        }
 
         // ---- combine the KPW key groups of the warp, write the partial ----
 #pragma unroll
