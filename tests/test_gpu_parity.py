@@ -2,7 +2,7 @@
 
 * the tiny sweep, exhaustively: every sequence, layer and step 0..T;
 * the hand-derived cases of tests/golden/hand_cases.json, zero-padded to d = 64;
-* edge shapes: ragged prompt spans, group sizes 1/2/3/8, d = 64/128/256,
+* edge shapes: ragged prompt spans, group sizes 1/2/3/4/6/8, d = 64/128/256,
   sliding windows shorter than the prompt span, a single sequence;
 * the four model-shaped sweeps at full size, in the launch configuration the
   bench times, on sampled (sequence, layer, step) outputs.
@@ -136,6 +136,14 @@ EDGE = [
     ("window_below_suffix", 3, 8, 2, 64, 1, 64, (WL.ZERO, WL.BLANK), 50, 20, 0),
     # five prompt-span splits: four of 3072 keys and a short last one
     ("long_span_5_splits", 1, 4, 2, 64, 1, 13000, (WL.SAME_ALGO, WL.ZERO), 3, 0, 0),
+    # generated-span pass at every (d, rows per item) it is built for, with
+    # generated spans long enough for several key splits and a ragged block:
+    # one row per item at d = 128 and 256 (fewer logits per key group than
+    # lanes), two rows (G = 6: three row chunks), four rows at d = 256
+    ("g1_d128_long_suffix", 2, 4, 4, 128, 1, 150, (WL.BLANK, WL.ZERO), 150, 0, 0),
+    ("g6_d128_long_suffix", 2, 12, 2, 128, 1, 97, (WL.DIFF_ALGO, WL.ZERO), 150, 0, 0),
+    ("g4_d256_long_suffix", 2, 8, 2, 256, 1, 140, (WL.SAME_ALGO, WL.ZERO), 150, 0, 0),
+    ("g1_d256_long_suffix", 2, 2, 2, 256, 1, 90, (WL.DIFF_FAMILY, WL.ZERO), 150, 0, 0),
 ]
 
 
