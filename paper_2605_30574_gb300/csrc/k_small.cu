@@ -30,13 +30,13 @@ __global__ void append_kernel(const uint4* __restrict__ kn, const uint4* __restr
     vs[dst] = vn[i];
 }
 
-// One warp per output row: the partial states of the prompt-span and the
-// generated-span passes (and the ZERO closed form) -> out.  Rows with up to
-// four partials -- the common case -- take the one-round-trip path, whose
-// few registers let six blocks (48 warps) share an SM, so more rows' loads
-// are in flight at once.
+// The partial states of the prompt-span and the generated-span passes (and
+// the ZERO closed form) -> out.  Rows with up to four partials -- the common
+// case -- take a one-round-trip path: for d <= 128 a warp merges two rows,
+// one per half-warp; for d = 256 one row per warp.  Rows with more partials
+// take the general path, a warp per row.
 template <int D>
-__global__ void __launch_bounds__(256, 6) merge_kernel(AttnParams P) {
+__global__ void __launch_bounds__(256, D <= 128 ? 5 : 6) merge_kernel(AttnParams P) {
     // Launched behind the prompt-span pass as a programmatic dependent, this
     // grid may start before that pass has finished: wait for it (and so for
     // the generated-span pass it waited for) before reading any partial.
@@ -44,8 +44,17 @@ __global__ void __launch_bounds__(256, 6) merge_kernel(AttnParams P) {
     asm volatile("griddepcontrol.wait;" ::: "memory");
     const long warp = (long(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
-    if (warp >= long(P.B) * P.Hq) return;
-    if (!merge_row_fast<D, 4>(P, warp, lane)) merge_row(P, warp, lane);
+    const long total = long(P.B) * P.Hq;
+    if constexpr (D <= 128) {
+        const long row0 = 2 * warp;
+        if (row0 >= total) return;
+        if (merge_rows_fast2<D, 4>(P, row0, lane)) return;
+        merge_row(P, row0, lane);
+        if (row0 + 1 < total) merge_row(P, row0 + 1, lane);
+    } else {
+        if (warp >= total) return;
+        if (!merge_row_fast<D, 4>(P, warp, lane)) merge_row(P, warp, lane);
+    }
 }
 
 }  // namespace
@@ -65,7 +74,8 @@ int launch_append(const uint16_t* kn, const uint16_t* vn, uint16_t* ks, uint16_t
 int launch_merge(const AttnParams& p, void* stream, bool overlap_previous) {
     const long rows = long(p.B) * p.Hq;
     const int block = 256;
-    const long threads = rows * 32;
+    const long warps = p.D <= 128 ? (rows + 1) / 2 : rows;
+    const long threads = warps * 32;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(unsigned((threads + block - 1) / block));
     cfg.blockDim = dim3(block);

@@ -51,7 +51,7 @@ __device__ __forceinline__ float merge_weights(const AttnParams& P, int lane, in
     float den = w * l;
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) den += __shfl_xor_sync(0xffffffffu, den, off);
-    if (zero_span) den += float(P.p_hi - P.p_lo) * exp2f(0.f - M);
+    if (zero_span) den = fmaf(float(P.p_hi - P.p_lo), exp2f(0.f - M), den);
     *w_out = w;
     return den > 0.f ? 1.f / den : 0.f;
 }
@@ -104,6 +104,81 @@ __device__ __forceinline__ bool merge_row_fast(const AttnParams& P, long row, in
     for (int q = 0; q < SL; ++q) {
         const int c = lane + 32 * q;
         if (c < C4) out[c] = make_float4(acc[q].x * inv, acc[q].y * inv, acc[q].z * inv, acc[q].w * inv);
+    }
+    return true;
+}
+
+// Two rows per warp, one per half-warp (lanes 0-15 row0, 16-31 row0 + 1),
+// for rows of at most NF live partials each: the loads of both rows go out
+// at once, twice the rows in flight per warp.  The reductions run over the
+// 16 lanes of a half with the partials on lanes 0 .. n-1 of it, so they add
+// the same values in the same order as merge_weights over 32 lanes (the
+// other lanes hold zeros): the same bits as merge_row_fast.  False (nothing
+// written) if either row has more partials.
+template <int D, int NF>
+__device__ __forceinline__ bool merge_rows_fast2(const AttnParams& P, long row0, int lane) {
+    constexpr int C4 = D / 4;                    // float4 slices of a row
+    constexpr int SL = (C4 + 15) / 16;           // slices per lane of a half
+    const int half = lane >> 4, hl = lane & 15;
+    const long total = long(P.B) * P.Hq;
+    const long row = row0 + half;
+    const bool live_row = row < total;
+    RowParts rp{0, 0, 0};
+    uint8_t code = SPLICE_SRC_CLEAN;
+    if (live_row) {
+        code = P.src[int(row / P.Hq)];
+        rp = row_parts(P, code);
+    }
+    const int n = rp.span + rp.suffix + rp.delta;
+    if (!__all_sync(0xffffffffu, n <= NF)) return false;
+    const size_t plane = size_t(total);
+    float2 ml = make_float2(-INFINITY, 0.f);
+    if (hl < n) ml = __ldcg(P.ws_ml + size_t(merge_slot(hl, rp)) * plane + row);
+    float4 ov[NF][SL];
+#pragma unroll
+    for (int i = 0; i < NF; ++i) {
+        const float4* src = reinterpret_cast<const float4*>(P.ws_o + (size_t(merge_slot(i, rp)) * plane + row) * D);
+#pragma unroll
+        for (int q = 0; q < SL; ++q) {
+            const int c = hl + 16 * q;
+            ov[i][q] = (i < n && c < C4) ? __ldcg(src + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+    }
+    // weights over the half: as merge_weights
+    const bool zero_span = code == SPLICE_SRC_ZERO && P.p_hi > P.p_lo;
+    float M = (hl < n && ml.y > 0.f) ? ml.x : -INFINITY;
+    if (zero_span) M = fmaxf(M, 0.f);
+#pragma unroll
+    for (int off = 8; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    const float w = (hl < n && ml.y > 0.f) ? exp2f(ml.x - M) : 0.f;
+    float den = w * ml.y;
+#pragma unroll
+    for (int off = 8; off > 0; off >>= 1) den += __shfl_xor_sync(0xffffffffu, den, off);
+    if (zero_span) den = fmaf(float(P.p_hi - P.p_lo), exp2f(0.f - M), den);
+    const float inv = den > 0.f ? 1.f / den : 0.f;
+    float4 acc[SL];
+#pragma unroll
+    for (int q = 0; q < SL; ++q) acc[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int i = 0; i < NF; ++i) {
+        const float wi = __shfl_sync(0xffffffffu, w, (half << 4) + i);
+        if (i < n && wi != 0.f) {
+#pragma unroll
+            for (int q = 0; q < SL; ++q) {
+                acc[q].x = fmaf(wi, ov[i][q].x, acc[q].x);
+                acc[q].y = fmaf(wi, ov[i][q].y, acc[q].y);
+                acc[q].z = fmaf(wi, ov[i][q].z, acc[q].z);
+                acc[q].w = fmaf(wi, ov[i][q].w, acc[q].w);
+            }
+        }
+    }
+    if (live_row) {
+        float4* out = reinterpret_cast<float4*>(P.out + size_t(row) * D);
+#pragma unroll
+        for (int q = 0; q < SL; ++q) {
+            const int c = hl + 16 * q;
+            if (c < C4) out[c] = make_float4(acc[q].x * inv, acc[q].y * inv, acc[q].z * inv, acc[q].w * inv);
+        }
     }
     return true;
 }
