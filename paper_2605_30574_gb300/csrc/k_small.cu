@@ -36,7 +36,7 @@ __global__ void append_kernel(const uint4* __restrict__ kn, const uint4* __restr
 // one per half-warp; for d = 256 one row per warp.  Rows with more partials
 // take the general path, a warp per row.
 template <int D>
-__global__ void __launch_bounds__(256, D <= 128 ? 5 : 6) merge_kernel(AttnParams P) {
+__global__ void __launch_bounds__(256, 5) merge_kernel(AttnParams P) {
     // Launched behind the prompt-span pass as a programmatic dependent, this
     // grid may start before that pass has finished: wait for it (and so for
     // the generated-span pass it waited for) before reading any partial.
