@@ -5,11 +5,13 @@ prompt span, 5 donor slots, 1024 decode steps, (L, W) grid 5 x 4, 512-sequence
 decode batches).
 
 One *step* = one decode step of one 512-sequence batch through all layers:
-per layer one ``suffix_kv_append`` and one ``spliced_decode_attn``.  Steps
-walk the decode steps t of the sweep in a stratified order (t_k at the
-midpoints of K equal slices of 1..T), so the mix of generated-span lengths and
-splice epochs matches the whole run.  The metric is sequence-steps per second
-(one sequence-step = all layers and heads of one sequence at one t).
+per layer one ``spliced_decode_step`` (the step's append done inside the
+generated-span pass, then the attention; ``--unfused``: ``suffix_kv_append``
++ ``spliced_decode_attn``).  Steps walk the decode steps t of the sweep in a
+stratified order (t_k at the midpoints of K equal slices of 1..T), so the mix
+of generated-span lengths and splice epochs matches the whole run.  The
+metric is sequence-steps per second (one sequence-step = all layers and heads
+of one sequence at one t).
 
 Legs (one JSON line on rank 0):
 * value: device-resident inputs, CUDA events around exactly K steps;
@@ -19,14 +21,18 @@ Legs (one JSON line on rank 0):
 * e2e: the same K steps through the C ABI with the step's queries and new
   K/V copied from pinned host memory and the outputs copied back, copies
   overlapped with compute on separate streams;
-* graph: each timed step's calls (every layer's append and attention)
-  captured once into a CUDA graph before the timed region, then the K graphs
-  replayed under the same events -- the fused-step launch mode;
+* graph: each timed step's calls (every layer) captured once into a CUDA
+  graph before the timed region, then the K graphs replayed under the same
+  events -- the fused-step launch mode;
 * delta: the same K steps in delta-donor mode (donor spans that share most
   positions with the clean span encoded against it once, before timing);
+* workloads: the Qwen3-4B-, Llama-3-8B- and Gemma-3-4B-shaped sweeps (batch
+  0, fewer steps), each with its own algorithmic bytes and kernel split;
 * cpu_baseline: the fp64 CPU oracle on a bounded sample of (sequence,
   layer, step) units of the same batch, on the host's cores.
 ``--impl reference`` times that oracle alone as the reference arm.
+``--profile-case`` runs one small, fixed launch sequence for profilers (see
+``profile_case``) instead of the bench.
 """
 from __future__ import annotations
 
@@ -90,8 +96,9 @@ def read_peaks():
 # --------------------------------------------------------------------------
 # algorithmic bytes (what the method must move), from the source maps
 # --------------------------------------------------------------------------
-def algorithmic_bytes(sb, layer: int, step: int, delta=None):
-    """Bytes per kernel kind at (layer, step).  ``delta`` = (slot flags,
+def algorithmic_bytes(sb, layer: int, step: int, delta=None, fused=False):
+    """Bytes per kernel kind at (layer, step) (``fused``: the step's append
+    runs inside the generated-span pass).  ``delta`` = (slot flags,
     encoded counts [prompts][stored slots][N][Hkv]) in delta mode: a reader
     of an encoded slot reads its prompt's clean span (shared with the clean
     readers) and the slot's encoded rows instead of the donor span."""
@@ -116,13 +123,16 @@ def algorithmic_bytes(sb, layer: int, step: int, delta=None):
             stq = sum(1 for j in range(k) if wl.slot_kinds[j] != 0)
             rows += int(delta[1][p - sb.p0, stq, layer].sum()) * wl.head_dim * 4
     n_span = sum(1 for _, code in spans if code >= 0)
-    n_read = sum(1 for code in m if code != S.SRC_ZERO)
     q_bytes = wl.num_q_heads * wl.head_dim * 2
+    append = sb.B * wl.num_kv_heads * wl.head_dim * 8 if step >= 1 else 0
+    # each sequence's q counted once (with the generated-span pass, which
+    # reads every sequence's q); in the fused call the append's bytes are
+    # moved by the generated-span pass
     return {
-        "prompt_span_pass": n_span * st["prompt_visible"] * kv_pos + rows + n_read * q_bytes,
-        "generated_span_pass": sb.B * st["suffix_visible"] * kv_pos + sb.B * q_bytes,
+        "prompt_span_pass": n_span * st["prompt_visible"] * kv_pos + rows,
+        "generated_span_pass": sb.B * st["suffix_visible"] * kv_pos + sb.B * q_bytes + (append if fused else 0),
         "merge": sb.B * wl.num_q_heads * wl.head_dim * 4,
-        "append": sb.B * wl.num_kv_heads * wl.head_dim * 8 if step >= 1 else 0,
+        "append": 0 if fused else append,
     }
 
 
@@ -231,22 +241,36 @@ def _oracle_worker(name, units, barrier, results):
     results.put((len(prepared), time.perf_counter() - t0))
 
 
-def run_oracle_sample(name, units_per_core, cores, seed, batch=0):
-    """Times the oracle on cores x units_per_core units (generation excluded)."""
-    import multiprocessing as mp
-    from paper_2605_30574_gb300.synth import workloads as W
-    wl = W.get(name)
-    rng = np.random.default_rng(seed)
+def plan_units(wl, batch, seed):
+    """(s, l, t) units of the parity sampling plan inside one sweep batch,
+    shuffled: every cell of the batch's first and last prompts at steps {1,
+    W - 1, W, W + 1, T / 2, T} of the cell's own onset, every layer."""
     lo, hi = wl.batch_range(batch)
-    ts = step_schedule(wl.max_steps, 16)
-    units = [[(int(rng.integers(lo, hi)), int(rng.integers(0, wl.num_layers)), int(ts[rng.integers(0, 16)]))
-              for _ in range(units_per_core)] for _ in range(cores)]
+    seqs = wl.sequences()
+    N, T = wl.num_layers, wl.max_steps
+    ends = {seqs[lo].prompt, seqs[hi - 1].prompt}
+    units = []
+    for s in range(lo, hi):
+        q = seqs[s]
+        if q.prompt not in ends:
+            continue
+        steps = sorted({x for x in (1, q.W - 1, q.W, q.W + 1, T // 2, T) if 1 <= x <= T})
+        units += [(s, l, t) for l in range(N) for t in steps]
+    rng = np.random.default_rng(seed)
+    rng.shuffle(units)
+    return units
+
+
+def run_oracle_sample(name, per_core):
+    """Times the oracle on per_core[c] units in process c (generation excluded);
+    returns (units, wall seconds of the slowest process)."""
+    import multiprocessing as mp
     for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
         os.environ[k] = "1"
     ctx = mp.get_context("spawn")
-    barrier = ctx.Barrier(cores + 1)
+    barrier = ctx.Barrier(len(per_core) + 1)
     results = ctx.Queue()
-    procs = [ctx.Process(target=_oracle_worker, args=(name, units[c], barrier, results)) for c in range(cores)]
+    procs = [ctx.Process(target=_oracle_worker, args=(name, units, barrier, results)) for units in per_core]
     for p in procs:
         p.start()
     barrier.wait()
@@ -255,24 +279,40 @@ def run_oracle_sample(name, units_per_core, cores, seed, batch=0):
     wall = time.perf_counter() - t0
     for p in procs:
         p.join()
-    n_units = sum(g[0] for g in got)
-    return n_units, wall
+    return sum(g[0] for g in got), wall
 
 
-def cpu_baseline(name, budget_s=15.0):
+def host_cores():
+    """(cores the oracle uses = the CPUs this process may run on, os.cpu_count())."""
+    try:
+        aff = len(os.sched_getaffinity(0))
+    except AttributeError:      # pragma: no cover
+        aff = os.cpu_count() or 1
+    return max(1, aff), os.cpu_count() or 1
+
+
+def cpu_baseline(name, budget_s=15.0, batch=0):
     from paper_2605_30574_gb300.synth import workloads as W
     wl = W.get(name)
-    cores = max(1, min(os.cpu_count() or 1, 16))
-    # calibrate: one unit on one core
-    n1, w1 = run_oracle_sample(name, 1, 1, seed=99)
+    cores, n_cpu = host_cores()
+    units = plan_units(wl, batch, seed=7)
+    # one thread: a few units alone
+    n1, w1 = run_oracle_sample(name, [units[:3]])
     per_unit = w1 / max(n1, 1)
     upc = int(max(1, min(64, budget_s / per_unit)))
-    n, wall = run_oracle_sample(name, upc, cores, seed=7)
+    need = cores * upc
+    take = (units * (need // len(units) + 1))[:need]
+    n, wall = run_oracle_sample(name, [take[c::cores] for c in range(cores)])
     value = n / wall / wl.num_layers
-    return {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
-            "sample": (f"{n} (sequence, layer, step) units of batch 0 ({upc} per core, random layer, steps at "
-                       f"16 stratified t), fp64 numpy oracle, input generation excluded; "
-                       f"{wall:.1f} s wall; seq-steps = units / {wl.num_layers} layers")}
+    return {"value": value, "unit": UNIT, "cores": cores, "os_cpu_count": n_cpu, "affinity_cores": cores,
+            "value_1thread": 1.0 / per_unit / wl.num_layers, "kind": "oracle",
+            "sample": (f"{n} (sequence, layer, step) units of batch {batch} from the parity sampling plan (every "
+                       f"cell of the batch's first and last prompts at steps 1, W-1, W, W+1, T/2, T of its own "
+                       f"onset, every layer; {upc} per core), fp64 numpy oracle, input generation excluded; "
+                       f"{wall:.1f} s wall on {cores} processes; seq-steps = units / {wl.num_layers} layers; "
+                       f"value_1thread from {n1} units on one core"),
+            "note": ("a plain per-head fp64 numpy loop, deliberately slow: the GPU/CPU ratio says nothing about "
+                     "kernel quality (the roofline fraction does)")}
 
 
 def reference_arm(args):
@@ -281,12 +321,14 @@ def reference_arm(args):
         return 0
     from paper_2605_30574_gb300.synth import workloads as W
     wl = W.get(args.workload)
-    cores = max(1, min(os.cpu_count() or 1, 16))
+    cores, n_cpu = host_cores()
+    units = plan_units(wl, args.batch, seed=11)
+    per_step = [units[(k * cores + c) % len(units)] for k in range(args.warmup + args.steps) for c in range(cores)]
     for w in range(args.warmup):
-        run_oracle_sample(args.workload, 1, cores, seed=1000 + w)
+        run_oracle_sample(args.workload, [[u] for u in per_step[w * cores:(w + 1) * cores]])
     total_units, total_wall = 0, 0.0
-    for k in range(args.steps):
-        n, wall = run_oracle_sample(args.workload, 1, cores, seed=k)
+    for k in range(args.warmup, args.warmup + args.steps):
+        n, wall = run_oracle_sample(args.workload, [[u] for u in per_step[k * cores:(k + 1) * cores]])
         total_units += n
         total_wall += wall
     value = total_units / total_wall / wl.num_layers
@@ -295,9 +337,9 @@ def reference_arm(args):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic",
             "config": {"workload": describe(wl), "batch": wl.batch},
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
-                             "sample": f"each step: {cores} random (sequence, layer, step) units of batch 0, "
-                                       f"one per core; input generation excluded"},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "os_cpu_count": n_cpu, "kind": "oracle",
+                             "sample": f"each step: {cores} (sequence, layer, step) units of batch {args.batch} "
+                                       f"from the parity sampling plan, one per core; input generation excluded"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
     return 0
@@ -312,13 +354,75 @@ def describe(wl):
 # --------------------------------------------------------------------------
 # GPU arm
 # --------------------------------------------------------------------------
+def make_run_step(sb, fused: bool):
+    """One decode step of the whole batch through every layer, on a stream."""
+    from paper_2605_30574_gb300 import splice as S
+    N = sb.wl.num_layers
+
+    def run_step(t, q, k_new, v_new, out, st):
+        for l in range(N):
+            if fused:
+                S.spliced_decode_step(sb.desc, l, t, q[l], k_new[l], v_new[l], sb.k_clean, sb.v_clean, sb.k_donor,
+                                      sb.v_donor, sb.k_suffix, sb.v_suffix, out[l], sb.ws, stream=st)
+            else:
+                S.suffix_kv_append(sb.desc, l, t, k_new[l], v_new[l], sb.k_suffix, sb.v_suffix, st)
+                S.spliced_decode_attn(sb.desc, l, t, q[l], sb.k_clean, sb.v_clean, sb.k_donor, sb.v_donor,
+                                      sb.k_suffix, sb.v_suffix, out[l], sb.ws, stream=st)
+    return run_step
+
+
+def gen_step_inputs(sb, ts, dev):
+    """Queries and new K/V of every layer of steps ts, generated ahead (excluded from timing)."""
+    import torch
+    from paper_2605_30574_gb300.synth import device as SD
+    wl, N = sb.wl, sb.wl.num_layers
+    qs = torch.empty((len(ts), N) + tuple(sb.q.shape), dtype=torch.bfloat16, device=dev)
+    kn = torch.empty((len(ts), N) + tuple(sb.k_new.shape), dtype=torch.bfloat16, device=dev)
+    vn = torch.empty_like(kn)
+    for i, t in enumerate(ts):
+        for l in range(N):
+            SD.fill_q(wl, sb.s0, l, t, qs[i, l])
+            SD.fill_new_kv(wl, sb.s0, l, t, kn[i, l], vn[i, l])
+    return qs, kn, vn
+
+
+def profile_pass(sb, steps, qs, kn, vn, outs, run_step, stream):
+    """The same steps with the library's per-launch events: {kind: (launches, ms)}."""
+    import torch
+    from paper_2605_30574_gb300 import splice as S
+    S.splice_profile_enable(sb.desc, True)
+    S.splice_profile_read(sb.desc)
+    torch.cuda.synchronize()
+    for i, t in enumerate(steps):
+        run_step(t, qs[i], kn[i], vn[i], outs, stream)
+    torch.cuda.synchronize()
+    prof = S.splice_profile_read(sb.desc)
+    S.splice_profile_enable(sb.desc, False)
+    return prof
+
+
+def kernel_table(prof, per_kind):
+    total = sum(x[1] for x in prof.values()) or 1.0
+    return {k: {"launches": v[0], "ms_total": round(v[1], 3), "share": round(v[1] / total, 4),
+                "GBps": round(per_kind[k] / (v[1] / 1000.0) / 1e9, 1) if v[1] > 0 else None}
+            for k, v in prof.items()}
+
+
+def step_bytes(sb, steps, fused):
+    per_kind = {"append": 0, "prompt_span_pass": 0, "generated_span_pass": 0, "merge": 0}
+    for t in steps:
+        for l in range(sb.wl.num_layers):
+            for k, v in algorithmic_bytes(sb, l, t, fused=fused).items():
+                per_kind[k] += v
+    return per_kind
+
+
 def gpu_arm(args):
     import torch
     import torch.distributed as dist
     from paper_2605_30574_gb300 import build as B
     from paper_2605_30574_gb300 import splice as S
     from paper_2605_30574_gb300.sweep import SweepBatch
-    from paper_2605_30574_gb300.synth import device as SD
     from paper_2605_30574_gb300.synth import workloads as W
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -328,6 +432,7 @@ def gpu_arm(args):
         dist.init_process_group("nccl")
     torch.cuda.set_device(local)
     B.build()
+    fused = not args.unfused
     wl = W.get(args.workload)
     batch = rank_batch(wl.num_batches(), args.batch, rank)
     sb = SweepBatch(wl, batch)
@@ -335,31 +440,14 @@ def gpu_arm(args):
     steps = step_schedule(wl.max_steps, args.steps)
     warm = step_schedule(wl.max_steps, max(args.warmup, 1), offset=0)[: args.warmup]
     dev = torch.device("cuda", local)
-    # this step's inputs for every layer, generated ahead (excluded from timing)
-    def gen(ts):
-        qs = torch.empty((len(ts), N) + tuple(sb.q.shape), dtype=torch.bfloat16, device=dev)
-        kn = torch.empty((len(ts), N) + tuple(sb.k_new.shape), dtype=torch.bfloat16, device=dev)
-        vn = torch.empty_like(kn)
-        for i, t in enumerate(ts):
-            for l in range(N):
-                SD.fill_q(wl, sb.s0, l, t, qs[i, l])
-                SD.fill_new_kv(wl, sb.s0, l, t, kn[i, l], vn[i, l])
-        return qs, kn, vn
-
-    qs, kn, vn = gen(steps)
-    wq, wkn, wvn = gen(warm) if warm else (None, None, None)
+    qs, kn, vn = gen_step_inputs(sb, steps, dev)
+    wq, wkn, wvn = gen_step_inputs(sb, warm, dev) if warm else (None, None, None)
     outs = torch.empty((N,) + tuple(sb.out.shape), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream()
-
-    def run_step(t, q, k_new, v_new, out, st=None):
-        st = stream if st is None else st
-        for l in range(N):
-            S.suffix_kv_append(sb.desc, l, t, k_new[l], v_new[l], sb.k_suffix, sb.v_suffix, st)
-            S.spliced_decode_attn(sb.desc, l, t, q[l], sb.k_clean, sb.v_clean, sb.k_donor, sb.v_donor,
-                                  sb.k_suffix, sb.v_suffix, out[l], sb.ws, stream=st)
+    run_step = make_run_step(sb, fused)
 
     for i, t in enumerate(warm):
-        run_step(t, wq[i], wkn[i], wvn[i], outs)
+        run_step(t, wq[i], wkn[i], wvn[i], outs, stream)
     torch.cuda.synchronize()
 
     # ---- value: exactly K steps, device-resident inputs ----
@@ -371,7 +459,7 @@ def gpu_arm(args):
     with ClockSampler(local) as clk:
         ev0.record(stream)
         for i, t in enumerate(steps):
-            run_step(t, qs[i], kn[i], vn[i], outs)
+            run_step(t, qs[i], kn[i], vn[i], outs, stream)
         ev1.record(stream)
         torch.cuda.synchronize()
     if world > 1:
@@ -384,30 +472,15 @@ def gpu_arm(args):
     ms, units = reduce_timing(ms, units, dist if world > 1 else None, dev)
     value = units / (ms / 1000.0)
 
-    # ---- algorithmic bytes of the timed steps ----
-    per_kind = {"append": 0, "prompt_span_pass": 0, "generated_span_pass": 0, "merge": 0}
-    for t in steps:
-        for l in range(N):
-            for k, v in algorithmic_bytes(sb, l, t).items():
-                per_kind[k] += v
+    # ---- algorithmic bytes of the timed steps, and the roofline pass ----
+    per_kind = step_bytes(sb, steps, fused)
     total_bytes = sum(per_kind.values())
-
-    # ---- roofline pass: per-launch events recorded by the library ----
-    S.splice_profile_enable(sb.desc, True)
-    S.splice_profile_read(sb.desc)
-    torch.cuda.synchronize()
-    for i, t in enumerate(steps):
-        run_step(t, qs[i], kn[i], vn[i], outs)
-    torch.cuda.synchronize()
-    prof = S.splice_profile_read(sb.desc)
-    S.splice_profile_enable(sb.desc, False)
+    prof = profile_pass(sb, steps, qs, kn, vn, outs, run_step, stream)
     peak, peak_kind = read_peaks()
     dom = max(prof, key=lambda k: prof[k][1])
     n_l, ms_l = prof[dom]
     achieved = (per_kind[dom] / max(n_l, 1)) / ((ms_l / max(n_l, 1)) / 1000.0) / 1e9
-    kernels = {k: {"launches": v[0], "ms_total": round(v[1], 3), "share": round(v[1] / sum(x[1] for x in prof.values()), 4),
-                   "GBps": round(per_kind[k] / (v[1] / 1000.0) / 1e9, 1) if v[1] > 0 else None}
-               for k, v in prof.items()}
+    kernels = kernel_table(prof, per_kind)
 
     # ---- graph: every timed step captured once, then replayed ----
     graph = None
@@ -417,22 +490,33 @@ def gpu_arm(args):
     # ---- delta: donor spans encoded against the clean spans ----
     delta = None
     if not args.no_delta and sb.Dst:
-        delta = delta_leg(sb, steps, qs, kn, vn, outs, run_step, world, dist, per_kind)
+        delta = delta_leg(sb, steps, qs, kn, vn, outs, run_step, world, dist, per_kind, fused)
 
     # ---- e2e: host buffers through the C ABI, copies overlapped ----
     e2e = None
     if not args.no_e2e:
         e2e = e2e_leg(sb, steps, qs, kn, vn, run_step, dev)
-    del qs, kn, vn
+    del qs, kn, vn, wq, wkn, wvn, outs
+    sb.close()
+    del sb
+    torch.cuda.empty_cache()
+
+    # ---- the other model-shaped sweeps ----
+    workloads = None
+    if not args.no_workloads and rank == 0 and world == 1:
+        workloads = {name: workload_leg(name, args.workload_steps, fused, dev, peak)
+                     for name in ("qwen3-4b", "llama3-8b", "gemma3-4b") if name != args.workload}
 
     if rank == 0:
-        cpu = None if args.no_cpu_baseline else cpu_baseline(args.workload)
+        cpu = None if args.no_cpu_baseline else cpu_baseline(args.workload, batch=batch)
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": len(steps),
             "warmup": args.warmup, "ms_per_step": ms / len(steps), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": describe(wl), "batch": f"batch {batch} of {wl.num_batches()}: sequences "
-                                                           f"{sb.s0}-{sb.s0 + sb.B - 1}",
+                                                           f"{wl.batch_range(batch)[0]}-{wl.batch_range(batch)[1] - 1}",
+                       "call": "spliced_decode_step (append fused into the generated-span pass)" if fused
+                               else "suffix_kv_append + spliced_decode_attn",
                        "decode_steps_t": steps, "l2": "inputs larger than L2 (every step streams >10 GB); no flush",
                        "parallelism": f"{world} GPU(s), one sweep batch each, no collective"},
             "hbm": {"algorithmic_GB_per_step": round(total_bytes / len(steps) / 1e9, 3),
@@ -446,13 +530,60 @@ def gpu_arm(args):
                          "bytes_per_launch": per_kind[dom] // max(n_l, 1),
                          "ms_per_launch": ms_l / max(n_l, 1)},
             "kernels": kernels,
-            "e2e": e2e, "graph": graph, "delta": delta, "gpu_launches": gpu_launches, "clocks": clk.summary(),
-            "cpu_baseline": cpu,
+            "e2e": e2e, "graph": graph, "delta": delta, "workloads": workloads, "gpu_launches": gpu_launches,
+            "clocks": clk.summary(), "cpu_baseline": cpu,
         }
         print(json.dumps(line))
     if world > 1:
         dist.destroy_process_group()
     return 0
+
+
+def workload_leg(name, n_steps, fused, dev, peak, warmup=2):
+    """One of the other model-shaped sweeps: batch 0, n_steps stratified
+    steps (the same timing rules), its algorithmic bytes and kernel split."""
+    import torch
+    from paper_2605_30574_gb300 import splice as S
+    from paper_2605_30574_gb300.sweep import SweepBatch
+    from paper_2605_30574_gb300.synth import workloads as W
+    wl = W.get(name)
+    sb = SweepBatch(wl, 0)
+    steps = step_schedule(wl.max_steps, n_steps)
+    warm = step_schedule(wl.max_steps, warmup)
+    qs, kn, vn = gen_step_inputs(sb, steps, dev)
+    wq, wkn, wvn = gen_step_inputs(sb, warm, dev)
+    outs = torch.empty((wl.num_layers,) + tuple(sb.out.shape), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+    run_step = make_run_step(sb, fused)
+    for i, t in enumerate(warm):
+        run_step(t, wq[i], wkn[i], wvn[i], outs, stream)
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(dev.index or 0) as clk:
+        ev0.record(stream)
+        for i, t in enumerate(steps):
+            run_step(t, qs[i], kn[i], vn[i], outs, stream)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    ms = ev0.elapsed_time(ev1)
+    S.splice_check_device_error(sb.desc)
+    per_kind = step_bytes(sb, steps, fused)
+    total = sum(per_kind.values())
+    prof = profile_pass(sb, steps, qs, kn, vn, outs, run_step, stream)
+    ideal = peak * 1e9 / (total / len(steps)) * sb.B
+    value = sb.B * len(steps) / (ms / 1000.0)
+    out = {"workload": describe(wl), "batch": f"batch 0: {sb.B} sequences", "steps": len(steps),
+           "decode_steps_t": steps, "value": value, "unit": UNIT, "ms_per_step": ms / len(steps),
+           "algorithmic_GB_per_step": round(total / len(steps) / 1e9, 3),
+           "achieved_GBps": round(total / (ms / 1000.0) / 1e9, 1),
+           "frac_of_measured": round(total / (ms / 1000.0) / 1e9 / peak, 4),
+           "ideal_seq_steps_per_s_at_measured_peak": round(ideal, 1),
+           "kernels": kernel_table(prof, per_kind), "clocks": clk.summary()}
+    del qs, kn, vn, wq, wkn, wvn, outs
+    sb.close()
+    del sb
+    torch.cuda.empty_cache()
+    return out
 
 
 def graph_leg(sb, steps, qs, kn, vn, outs, run_step, world, dist):
@@ -464,7 +595,7 @@ def graph_leg(sb, steps, qs, kn, vn, outs, run_step, world, dist):
     for i, t in enumerate(steps):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g):
-            run_step(t, qs[i], kn[i], vn[i], outs, st=torch.cuda.current_stream())
+            run_step(t, qs[i], kn[i], vn[i], outs, torch.cuda.current_stream())
         graphs.append(g)
     for g in graphs[:3]:
         g.replay()
@@ -490,7 +621,7 @@ def graph_leg(sb, steps, qs, kn, vn, outs, run_step, world, dist):
                    "the timed region; the K graphs replayed under CUDA events"}
 
 
-def delta_leg(sb, steps, qs, kn, vn, outs, run_step, world, dist, plain_bytes, max_fraction=0.6):
+def delta_leg(sb, steps, qs, kn, vn, outs, run_step, world, dist, plain_bytes, fused, max_fraction=0.6):
     """The K timed steps in delta-donor mode: the batch's stored donor spans
     encoded against the clean spans once, before the timed region (slots
     whose encoded fraction is at most max_fraction), then the same steps
@@ -510,17 +641,18 @@ def delta_leg(sb, steps, qs, kn, vn, outs, run_step, world, dist, plain_bytes, m
     count_off = (spans * w32 * 4 + 255) // 256 * 256
     counts = buf[count_off: count_off + spans * 4].view(torch.int32).cpu().numpy().reshape(
         sb.Pl, sb.Dst, N, wl.num_kv_heads)
+    stream = torch.cuda.current_stream()
     for i, t in enumerate(steps[:2]):
-        run_step(t, qs[i], kn[i], vn[i], outs)
+        run_step(t, qs[i], kn[i], vn[i], outs, stream)
     torch.cuda.synchronize()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
-    ev0.record()
+    ev0.record(stream)
     for i, t in enumerate(steps):
-        run_step(t, qs[i], kn[i], vn[i], outs)
-    ev1.record()
+        run_step(t, qs[i], kn[i], vn[i], outs, stream)
+    ev1.record(stream)
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
@@ -529,15 +661,9 @@ def delta_leg(sb, steps, qs, kn, vn, outs, run_step, world, dist, plain_bytes, m
     per_kind = {"append": 0, "prompt_span_pass": 0, "generated_span_pass": 0, "merge": 0}
     for t in steps:
         for l in range(N):
-            for k, v in algorithmic_bytes(sb, l, t, (flags, counts)).items():
+            for k, v in algorithmic_bytes(sb, l, t, (flags, counts), fused=fused).items():
                 per_kind[k] += v
-    S.splice_profile_enable(sb.desc, True)
-    S.splice_profile_read(sb.desc)
-    for i, t in enumerate(steps):
-        run_step(t, qs[i], kn[i], vn[i], outs)
-    torch.cuda.synchronize()
-    prof = S.splice_profile_read(sb.desc)
-    S.splice_profile_enable(sb.desc, False)
+    prof = profile_pass(sb, steps, qs, kn, vn, outs, run_step, stream)
     S.splice_delta_clear(sb.desc)
     del buf
     units = sb.B * len(steps)
@@ -596,7 +722,7 @@ def e2e_leg(sb, steps, qs, kn, vn, run_step, dev):
             comp.wait_event(in_ready[k])
             if k >= NB:
                 comp.wait_event(out_free[k - NB])             # output slot b copied out
-            run_step(t, d_q[b], d_kn[b], d_vn[b], d_out[b])
+            run_step(t, d_q[b], d_kn[b], d_vn[b], d_out[b], comp)
             comp_done[k].record(comp)
             with torch.cuda.stream(d2h):
                 d2h.wait_event(comp_done[k])
@@ -616,6 +742,42 @@ def e2e_leg(sb, steps, qs, kn, vn, run_step, dev):
                    "on two copy streams overlapped with compute (three device slots)"}
 
 
+def profile_case(args):
+    """A small, fixed launch sequence for profilers: one decode step of a
+    reduced copy of a sweep (same heads, head dim, prompt span, donor slots
+    and (L, W) grid shape, but few layers, a shorter generated-span store and
+    a smaller batch) so a capture holds a few GB on the device while every
+    launch still streams more than the 129 MB L2.  Repeated --reps times."""
+    import torch
+    from paper_2605_30574_gb300 import build as B
+    from paper_2605_30574_gb300 import splice as S
+    from paper_2605_30574_gb300.sweep import SweepBatch
+    from paper_2605_30574_gb300.synth import workloads as W
+    B.build()
+    base = W.get(args.workload)
+    layers = args.layers
+    Ls = tuple(sorted({min(layers, round(L * layers / base.num_layers)) for L in base.L_values}))
+    wl = W.Workload(base.name + "-prof", layers, base.num_q_heads, base.num_kv_heads, base.head_dim,
+                    base.num_prompts, base.prompt_len, base.slot_kinds, args.step + 8, Ls, base.W_values,
+                    base.scaffold_head, base.scaffold_tail, batch=args.batch_size,
+                    sliding_window=base.sliding_window, global_every=base.global_every, sm_scale=base.sm_scale)
+    sb = SweepBatch(wl, 0)
+    for _ in range(args.reps):
+        for l in range(wl.num_layers):
+            sb.gen_inputs(l, args.step)
+            if args.unfused:
+                sb.append(l, args.step)
+                sb.attn(l, args.step)
+            else:
+                sb.step(l, args.step)
+    torch.cuda.synchronize()
+    S.splice_check_device_error(sb.desc)
+    gb = (sb.k_suffix.numel() + sb.k_clean.numel() + (sb.k_donor.numel() if sb.k_donor is not None else 0)) * 4 / 1e9
+    print(f"profile case ok: {wl.name}, {sb.B} sequences, step {args.step}, {wl.num_layers} layers, "
+          f"{args.reps} reps, stores {gb:.2f} GB, {'unfused' if args.unfused else 'fused'} calls")
+    return 0
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -624,11 +786,21 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--batch", type=int, default=0)
+    ap.add_argument("--unfused", action="store_true", help="suffix_kv_append + spliced_decode_attn per layer")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--no-delta", action="store_true")
+    ap.add_argument("--no-workloads", action="store_true")
+    ap.add_argument("--workload-steps", type=int, default=8, help="timed steps of each other sweep")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile-case", action="store_true", help="run the small profiling case instead")
+    ap.add_argument("--layers", type=int, default=4, help="profile case: layers")
+    ap.add_argument("--batch-size", type=int, default=256, help="profile case: sequences")
+    ap.add_argument("--step", type=int, default=512, help="profile case: decode step")
+    ap.add_argument("--reps", type=int, default=3, help="profile case: repetitions")
     args = ap.parse_args(argv)
+    if args.profile_case:
+        return profile_case(args)
     if args.impl == "reference":
         return reference_arm(args)
     return gpu_arm(args)

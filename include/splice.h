@@ -191,6 +191,30 @@ splice_status spliced_decode_attn(splice_desc* desc, int layer, int step, const 
                                   void* stream);
 
 /*
+ * spliced_decode_step -- one layer of one decode step: suffix_kv_append of
+ * (k_new, v_new) at entry step - 1 followed by spliced_decode_attn (Algorithm
+ * 1's loop body: the forward pass appends the step's generated K/V, then
+ * attends over the prompt span and the step's generated entries, §3), in
+ * fewer launches.  The generated-span pass writes the new entries into the
+ * store itself and reads them from its registers, so no separate append
+ * kernel runs.
+ *
+ *   k_new, v_new        [num_seqs][Hkv][d] bf16, this step's entries of `layer`
+ *   k_suffix, v_suffix  generated-span store; slots 0 .. step-2 valid on entry,
+ *                       slot step-1 written by this call
+ *   other arguments     as spliced_decode_attn
+ *
+ * 1 <= step <= max_steps.  Outputs and the store afterwards are bit-identical
+ * to suffix_kv_append + spliced_decode_attn on the same inputs.
+ */
+splice_status spliced_decode_step(splice_desc* desc, int layer, int step, const splice_bf16* q,
+                                  const splice_bf16* k_new, const splice_bf16* v_new,
+                                  const splice_bf16* k_clean, const splice_bf16* v_clean,
+                                  const splice_bf16* k_donor, const splice_bf16* v_donor,
+                                  splice_bf16* k_suffix, splice_bf16* v_suffix, float* out,
+                                  void* workspace, size_t workspace_bytes, void* stream);
+
+/*
  * spliced_decode_attn_static -- spliced_decode_attn for callers that cannot
  * allocate device memory.  The paper has no counterpart; this is a
  * deployment convenience.
@@ -205,12 +229,17 @@ splice_status spliced_decode_attn(splice_desc* desc, int layer, int step, const 
  * (64 MiB) inside the library, which every GPU that loads the library holds
  * until the process exits.  This call allocates nothing.
  *
+ *   - The scratch used is the array of the descriptor's device (the device
+ *     it was created on, where its kernels run); q on another device is
+ *     rejected with SPLICE_EINVAL.
  *   - The first call on a device looks up that array's device address (with
- *     the tensors' device made current); make that first call before any
+ *     that device made current), and looks it up again after the device's
+ *     context changed (a cudaDeviceReset); make that first call before any
  *     stream capture.
  *   - A descriptor whose splice_workspace_bytes() exceeds
  *     SPLICE_STATIC_SCRATCH_BYTES is rejected with SPLICE_EINVAL (reduce the
  *     batch, or use spliced_decode_attn with a workspace).
+ *     splice_static_scratch_bytes() returns that limit as built.
  *   - Every call on a device shares the one array, and it keeps the last
  *     call's contents; nothing in it needs to start at zero.  Calls that
  *     overlap on the GPU (other streams, other host threads, other
@@ -219,6 +248,7 @@ splice_status spliced_decode_attn(splice_desc* desc, int layer, int step, const 
  * Arguments, layouts and errors are otherwise those of spliced_decode_attn.
  */
 #define SPLICE_STATIC_SCRATCH_BYTES (64u << 20)
+size_t splice_static_scratch_bytes(void);
 splice_status spliced_decode_attn_static(splice_desc* desc, int layer, int step, const splice_bf16* q,
                                          const splice_bf16* k_clean, const splice_bf16* v_clean,
                                          const splice_bf16* k_donor, const splice_bf16* v_donor,
@@ -349,6 +379,15 @@ const char* splice_kernel_kind_name(int kind);
  * bounded wait would; splice_check_device_error then returns SPLICE_EDEVICE.
  * Nothing faults or hangs. */
 splice_status splice_debug_wait_timeout(splice_desc* desc, unsigned limit_us, void* stream);
+
+/* Test of launch ordering: copies `bytes` (a multiple of 16; both pointers
+ * 16-byte aligned) from src to dst on `stream` with a kernel that lets its
+ * programmatic dependents launch as soon as it starts but copies only after
+ * delay_us microseconds (0 .. 1000000) of wall time.  A library call queued
+ * right behind it must still read the copied data: every kernel of the
+ * library waits for the work before it on the stream before it reads its
+ * inputs.  Nothing faults or hangs. */
+splice_status splice_debug_late_copy(void* dst, const void* src, size_t bytes, unsigned delay_us, void* stream);
 
 /* Static description of a status code. */
 const char* splice_status_str(splice_status status);

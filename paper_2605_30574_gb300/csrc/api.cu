@@ -51,9 +51,6 @@ struct splice_desc {
     std::vector<uint8_t> slot_delta;    // [Dslots]
     bool delta_on = false;
     char* delta = nullptr;
-    // (layer, step) of the append launched last, if it was the last launch
-    // through this descriptor (-1 otherwise)
-    int append_layer = -1, append_step = -1;
     int delta_max = 0;
     // TMA tensor maps of the clean and donor stores and of the delta rows
     // (K, V each), rebuilt when the store pointers change.
@@ -326,9 +323,172 @@ size_t workspace_bytes_of(const splice_desc* d) {
     return ml + o;
 }
 
+// One attention call: validation, the (epoch, layer class) table of (layer,
+// step), and the launches of the generated-span pass, the prompt-span pass
+// and the merge.  k_new / v_new non-NULL: the generated-span pass also
+// appends them at entry step - 1 (the fused decode step).
+splice_status attn_common(splice_desc* d, int layer, int step, const splice_bf16* q, const splice_bf16* k_new,
+                          const splice_bf16* v_new, const splice_bf16* k_clean, const splice_bf16* v_clean,
+                          const splice_bf16* k_donor, const splice_bf16* v_donor, splice_bf16* k_suffix,
+                          splice_bf16* v_suffix, float* out, void* workspace, size_t workspace_bytes, void* stream,
+                          const char* who) {
+    if (!d) return fail(SPLICE_EINVAL, "%s: descriptor is NULL", who);
+    if (!d->on_device) return fail(SPLICE_ESTATE, "%s: host-only descriptor", who);
+    if (layer < 0 || layer >= d->shape.num_layers) return fail(SPLICE_EINVAL, "%s: layer %d out of range", who, layer);
+    if (step < 0 || step > d->T) return fail(SPLICE_EINVAL, "%s: step %d not in [0, %d]", who, step, d->T);
+    if (!q || !k_clean || !v_clean || !out || !workspace)
+        return fail(SPLICE_EINVAL, "%s: NULL tensor or workspace", who);
+    if (step > 0 && (!k_suffix || !v_suffix)) return fail(SPLICE_EINVAL, "%s: NULL generated-span store", who);
+    if (d->Dst > 0 && (!k_donor || !v_donor)) return fail(SPLICE_EINVAL, "%s: NULL donor store", who);
+    const void* ptrs[] = {q, k_new, v_new, k_clean, v_clean, k_donor, v_donor, k_suffix, v_suffix, out, workspace};
+    for (const void* p : ptrs)
+        if (p && !aligned16(p)) return fail(SPLICE_EINVAL, "%s: tensor not 16-byte aligned", who);
+    if (workspace_bytes < workspace_bytes_of(d))
+        return fail(SPLICE_EINVAL, "%s: workspace of %zu bytes < %zu", who, workspace_bytes, workspace_bytes_of(d));
+    DeviceGuard g(d->device);
+    if (g.err != cudaSuccess) return cuda_fail(g.err, "cudaSetDevice");
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "earlier CUDA error");
+
+    const splice_model_shape& sh = d->shape;
+    const int tab = d->plan.table_of(layer, step);
+    const splice::Visible vis = splice::visible_keys(sh, d->Tp, layer, step);
+    const size_t rows = size_t(d->B) * sh.num_q_heads;
+    AttnParams p{};
+    p.q = q;
+    p.kc = k_clean;
+    p.vc = v_clean;
+    p.kd = k_donor;
+    p.vd = v_donor;
+    p.ks = k_suffix;
+    p.vs = v_suffix;
+    p.kn = k_new;
+    p.vn = v_new;
+    p.ks_w = k_suffix;
+    p.vs_w = v_suffix;
+    p.fuse_append = k_new ? 1 : 0;
+    p.out = out;
+    p.ws_ml = static_cast<float2*>(workspace);
+    p.ws_o = reinterpret_cast<float*>(static_cast<char*>(workspace) +
+                                      align_up(size_t(splice::kMaxSplits) * rows * sizeof(float2), 256));
+    p.src = d->d_src + size_t(tab) * d->B;
+    p.seq_prompt = d->d_seq_prompt;
+    p.seq_slot = d->d_seq_slot;
+    p.slot_stored = d->d_slot_stored;
+    p.tiles = d->d_tiles + 4 * size_t(d->plan.table_tile_off[tab]);
+    p.n_tiles = d->plan.table_tile_off[tab + 1] - d->plan.table_tile_off[tab];
+    p.group_prompt = d->d_group_prompt;
+    p.group_src = d->d_group_src;
+    p.group_seqs = d->d_group_seqs;
+    p.err = d->d_err;
+    p.sched = d->d_sched;
+    p.B = d->B;
+    p.N = sh.num_layers;
+    p.Hq = sh.num_q_heads;
+    p.Hkv = sh.num_kv_heads;
+    p.D = sh.head_dim;
+    p.G = sh.num_q_heads / sh.num_kv_heads;
+    p.Tp = d->Tp;
+    p.T = d->T;
+    p.Dst = d->Dst;
+    p.layer = layer;
+    p.step = step;
+    p.p_lo = vis.p_lo;
+    p.p_hi = vis.p_hi;
+    p.s_lo = vis.s_lo;
+    p.s_hi = vis.s_hi;
+    const int p_vis = vis.p_hi - vis.p_lo, s_vis = vis.s_hi - vis.s_lo;
+    // In delta mode a delta row's span splits and delta-row splits share the
+    // kMaxPrefixSplits prompt-span partial slots.
+    const int max_splits = d->delta_on ? splice::kMaxPrefixSplits / 2 : splice::kMaxPrefixSplits;
+    int tc_split = 0, tc_keys = 0;
+    int bounds[splice::kMaxPrefixSplits + 1] = {0};
+    if (p_vis > 0) {
+        tc_split = splice::prefix_tc_splits(sh.head_dim, p_vis, max_splits, bounds);
+        tc_keys = bounds[1];           // the longest split
+    }
+    p.nsp = tc_split;
+    p.n_span_tiles = d->plan.table_span_tiles[tab];
+    p.group_mask = d->d_group_mask;
+    p.slot_delta = d->d_slot_delta;
+    p.delta_on = d->delta_on ? 1 : 0;
+    p.nsd = 0;
+    if (d->delta_on) {
+        const DeltaLayout dl = delta_layout(d);
+        p.dmask = reinterpret_cast<const uint32_t*>(d->delta + dl.mask_off);
+        p.dcount = reinterpret_cast<const int32_t*>(d->delta + dl.count_off);
+        p.delta_w32 = dl.w32;
+        if (tc_keys > 0) p.nsd = std::min(max_splits, (d->delta_max + tc_keys - 1) / tc_keys);
+    }
+    {
+        // Generated-span items: (sequence, kv head, row chunk, key split).
+        // Split so every resident warp gets about two items, but keep at
+        // least 64 keys per split.  Every split costs a partial state to
+        // write and merge; the prompt-span pass queued behind this one fills
+        // the SMs its last warps leave idle, so few splits pay off even
+        // where the items do not share out evenly over the warps.
+        const int G = sh.num_q_heads / sh.num_kv_heads;
+        const int gt = G % 4 == 0 ? 4 : (G % 2 == 0 ? 2 : 1);
+        const long base_items = long(d->B) * sh.num_kv_heads * (G / gt);
+        const long want = 2L * splice::generated_span_resident_warps(sh.head_dim);
+        int ns = int(std::min<long>(splice::kMaxSuffixSplits, std::max<long>(1, (want + base_items - 1) / base_items)));
+        ns = std::min(ns, std::max(1, s_vis / 64));
+        p.nss = s_vis > 0 ? ns : 0;
+    }
+    p.p_chunk = tc_keys;
+    p.s_chunk = p.nss ? (s_vis + p.nss - 1) / p.nss : 0;
+    p.scale_log2 = sh.sm_scale * 1.4426950408889634f;
+
+    // The two passes read disjoint inputs and write disjoint partial slots.
+    // The generated-span pass goes first; the prompt-span pass is queued
+    // right behind it as a programmatic dependent launch, so its CTAs fill
+    // the SMs the generated-span pass's last CTAs leave idle, and it waits
+    // for that pass before it exits.  With per-launch timing on, the events
+    // between the launches serialise them instead.  (A fused call always has
+    // a generated span: step >= 1.)
+    const bool gs_launched = p.nss > 0;
+    if (gs_launched) {
+        e = timed_launch(d, 2, stream, [&] { return splice::launch_generated_span(p, stream, !d->profiling); });
+        if (e != cudaSuccess) return cuda_fail(e, "generated-span partials launch");
+    }
+    const long prefix_items = long(p.n_span_tiles) * sh.num_kv_heads * p.nsp +
+                              long(p.n_tiles - p.n_span_tiles) * sh.num_kv_heads * p.nsd;
+    const bool prefix_launched = p.nsp > 0 && prefix_items > 0;
+    if (prefix_launched) {
+        // Tensor maps over the stores viewed as [rows][d]; the delta rows
+        // have the donor store's layout.
+        const long rows_c = long(d->P) * sh.num_layers * sh.num_kv_heads * d->Tp;
+        const long rows_d = d->Dst ? rows_c * d->Dst : rows_c;
+        const DeltaLayout dl = delta_layout(d);
+        const void* xk = d->delta_on ? static_cast<const void*>(d->delta + dl.k_off) : k_clean;
+        const void* xv = d->delta_on ? static_cast<const void*>(d->delta + dl.v_off) : v_clean;
+        const void* mp[6] = {k_clean, v_clean, d->Dst ? k_donor : k_clean, d->Dst ? v_donor : v_clean, xk, xv};
+        const long mrows[6] = {rows_c, rows_c, rows_d, rows_d, d->delta_on ? rows_d : rows_c,
+                               d->delta_on ? rows_d : rows_c};
+        const int box = splice::prefix_tc_box_rows(sh.head_dim);
+        for (int i = 0; i < 6; ++i) {
+            if (d->map_ptr[i] == mp[i]) continue;
+            if (splice::make_kv_tensor_map(d->maps[i], mp[i], mrows[i], sh.head_dim, box) != 0)
+                return fail(SPLICE_ECUDA, "cuTensorMapEncodeTiled failed for store %d", i);
+            d->map_ptr[i] = mp[i];
+        }
+        const bool overlap = gs_launched && !d->profiling;
+        e = timed_launch(d, 1, stream, [&] {
+            return splice::launch_prefix_tc(p, d->maps, bounds, tc_keys, stream, overlap);
+        });
+        if (e != cudaSuccess) return cuda_fail(e, "prompt-span tensor-core pass launch");
+    }
+    const bool merge_overlap = prefix_launched && !d->profiling;
+    e = timed_launch(d, 3, stream, [&] { return splice::launch_merge(p, stream, merge_overlap); });
+    if (e != cudaSuccess) return cuda_fail(e, "merge launch");
+    return SPLICE_OK;
+}
+
 }  // namespace
 
 void splice::set_last_error(const char* msg) { g_last_error = msg; }
+
+int splice::desc_device(const splice_desc* d) { return d && d->on_device ? d->device : -1; }
 
 extern "C" {
 
@@ -412,14 +572,11 @@ splice_status suffix_kv_append(splice_desc* d, int layer, int step, const splice
     if (g.err != cudaSuccess) return cuda_fail(g.err, "cudaSetDevice");
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "earlier CUDA error");
-    d->append_layer = d->append_step = -1;
     e = timed_launch(d, 0, stream, [&] {
         return splice::launch_append(k_new, v_new, k_suffix, v_suffix, d->B, d->shape.num_layers,
                                      d->shape.num_kv_heads, d->shape.head_dim, d->T, layer, step, stream);
     });
     if (e != cudaSuccess) return cuda_fail(e, "append launch");
-    d->append_layer = layer;
-    d->append_step = step;
     return SPLICE_OK;
 }
 
@@ -428,155 +585,22 @@ splice_status spliced_decode_attn(splice_desc* d, int layer, int step, const spl
                                   const splice_bf16* k_donor, const splice_bf16* v_donor,
                                   const splice_bf16* k_suffix, const splice_bf16* v_suffix, float* out,
                                   void* workspace, size_t workspace_bytes, void* stream) {
-    if (!d) return fail(SPLICE_EINVAL, "descriptor is NULL");
-    if (!d->on_device) return fail(SPLICE_ESTATE, "host-only descriptor");
-    if (layer < 0 || layer >= d->shape.num_layers) return fail(SPLICE_EINVAL, "layer %d out of range", layer);
-    if (step < 0 || step > d->T) return fail(SPLICE_EINVAL, "step %d not in [0, %d]", step, d->T);
-    if (!q || !k_clean || !v_clean || !out || !workspace)
-        return fail(SPLICE_EINVAL, "NULL tensor or workspace");
-    if (step > 0 && (!k_suffix || !v_suffix)) return fail(SPLICE_EINVAL, "NULL generated-span store");
-    if (d->Dst > 0 && (!k_donor || !v_donor)) return fail(SPLICE_EINVAL, "NULL donor store");
-    const void* ptrs[] = {q, k_clean, v_clean, k_donor, v_donor, k_suffix, v_suffix, out, workspace};
-    for (const void* p : ptrs)
-        if (p && !aligned16(p)) return fail(SPLICE_EINVAL, "tensor not 16-byte aligned");
-    if (workspace_bytes < workspace_bytes_of(d))
-        return fail(SPLICE_EINVAL, "workspace of %zu bytes < %zu", workspace_bytes, workspace_bytes_of(d));
-    DeviceGuard g(d->device);
-    if (g.err != cudaSuccess) return cuda_fail(g.err, "cudaSetDevice");
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return cuda_fail(e, "earlier CUDA error");
+    return attn_common(d, layer, step, q, nullptr, nullptr, k_clean, v_clean, k_donor, v_donor,
+                       const_cast<splice_bf16*>(k_suffix), const_cast<splice_bf16*>(v_suffix), out, workspace,
+                       workspace_bytes, stream, "spliced_decode_attn");
+}
 
-    const splice_model_shape& sh = d->shape;
-    const int tab = d->plan.table_of(layer, step);
-    const splice::Visible vis = splice::visible_keys(sh, d->Tp, layer, step);
-    // The generated-span pass may read its older entries while the append
-    // launched right before it still runs, if that append wrote this layer
-    // and step (its only write is the entry this call reads last).
-    const bool dep_late = d->append_layer == layer && d->append_step == step && !d->profiling;
-    d->append_layer = d->append_step = -1;
-    const size_t rows = size_t(d->B) * sh.num_q_heads;
-    AttnParams p{};
-    p.q = q;
-    p.kc = k_clean;
-    p.vc = v_clean;
-    p.kd = k_donor;
-    p.vd = v_donor;
-    p.ks = k_suffix;
-    p.vs = v_suffix;
-    p.out = out;
-    p.ws_ml = static_cast<float2*>(workspace);
-    p.ws_o = reinterpret_cast<float*>(static_cast<char*>(workspace) +
-                                      align_up(size_t(splice::kMaxSplits) * rows * sizeof(float2), 256));
-    p.src = d->d_src + size_t(tab) * d->B;
-    p.seq_prompt = d->d_seq_prompt;
-    p.seq_slot = d->d_seq_slot;
-    p.slot_stored = d->d_slot_stored;
-    p.tiles = d->d_tiles + 4 * size_t(d->plan.table_tile_off[tab]);
-    p.n_tiles = d->plan.table_tile_off[tab + 1] - d->plan.table_tile_off[tab];
-    p.group_prompt = d->d_group_prompt;
-    p.group_src = d->d_group_src;
-    p.group_seqs = d->d_group_seqs;
-    p.err = d->d_err;
-    p.sched = d->d_sched;
-    p.B = d->B;
-    p.N = sh.num_layers;
-    p.Hq = sh.num_q_heads;
-    p.Hkv = sh.num_kv_heads;
-    p.D = sh.head_dim;
-    p.G = sh.num_q_heads / sh.num_kv_heads;
-    p.Tp = d->Tp;
-    p.T = d->T;
-    p.Dst = d->Dst;
-    p.layer = layer;
-    p.step = step;
-    p.p_lo = vis.p_lo;
-    p.p_hi = vis.p_hi;
-    p.s_lo = vis.s_lo;
-    p.s_hi = vis.s_hi;
-    const int p_vis = vis.p_hi - vis.p_lo, s_vis = vis.s_hi - vis.s_lo;
-    // In delta mode a delta row's span splits and delta-row splits share the
-    // kMaxPrefixSplits prompt-span partial slots.
-    const int max_splits = d->delta_on ? splice::kMaxPrefixSplits / 2 : splice::kMaxPrefixSplits;
-    int tc_split = 0, tc_keys = 0;
-    int bounds[splice::kMaxPrefixSplits + 1] = {0};
-    if (p_vis > 0) {
-        tc_split = splice::prefix_tc_splits(sh.head_dim, p_vis, max_splits, bounds);
-        tc_keys = bounds[1];           // the longest split
-    }
-    p.nsp = tc_split;
-    p.n_span_tiles = d->plan.table_span_tiles[tab];
-    p.group_mask = d->d_group_mask;
-    p.slot_delta = d->d_slot_delta;
-    p.delta_on = d->delta_on ? 1 : 0;
-    p.dep_late = dep_late ? 1 : 0;
-    p.nsd = 0;
-    if (d->delta_on) {
-        const DeltaLayout dl = delta_layout(d);
-        p.dmask = reinterpret_cast<const uint32_t*>(d->delta + dl.mask_off);
-        p.dcount = reinterpret_cast<const int32_t*>(d->delta + dl.count_off);
-        p.delta_w32 = dl.w32;
-        if (tc_keys > 0) p.nsd = std::min(max_splits, (d->delta_max + tc_keys - 1) / tc_keys);
-    }
-    {
-        // Generated-span items: (sequence, kv head, row chunk, key split).
-        // Split so every resident warp gets about two items, but keep at
-        // least 64 keys per split.  Every split costs a partial state to
-        // write and merge; the prompt-span pass queued behind this one fills
-        // the SMs its last warps leave idle, so few splits pay off even
-        // where the items do not share out evenly over the warps.
-        const int G = sh.num_q_heads / sh.num_kv_heads;
-        const int gt = G % 4 == 0 ? 4 : (G % 2 == 0 ? 2 : 1);
-        const long base_items = long(d->B) * sh.num_kv_heads * (G / gt);
-        const long want = 2L * splice::generated_span_resident_warps(sh.head_dim);
-        int ns = int(std::min<long>(splice::kMaxSuffixSplits, std::max<long>(1, (want + base_items - 1) / base_items)));
-        ns = std::min(ns, std::max(1, s_vis / 64));
-        p.nss = s_vis > 0 ? ns : 0;
-    }
-    p.p_chunk = tc_keys;
-    p.s_chunk = p.nss ? (s_vis + p.nss - 1) / p.nss : 0;
-    p.scale_log2 = sh.sm_scale * 1.4426950408889634f;
-
-    // The two passes read disjoint inputs and write disjoint partial slots.
-    // The generated-span pass goes first; the prompt-span pass is queued
-    // right behind it as a programmatic dependent launch, so its CTAs fill
-    // the SMs the generated-span pass's last CTAs leave idle, and it waits
-    // for that pass before it exits.  With per-launch timing on, the events
-    // between the launches serialise them instead.
-    const bool gs_launched = p.nss > 0;
-    if (gs_launched) {
-        e = timed_launch(d, 2, stream, [&] { return splice::launch_generated_span(p, stream, !d->profiling); });
-        if (e != cudaSuccess) return cuda_fail(e, "generated-span partials launch");
-    }
-    const long prefix_items = long(p.n_span_tiles) * sh.num_kv_heads * p.nsp +
-                              long(p.n_tiles - p.n_span_tiles) * sh.num_kv_heads * p.nsd;
-    const bool prefix_launched = p.nsp > 0 && prefix_items > 0;
-    if (prefix_launched) {
-        // Tensor maps over the stores viewed as [rows][d]; the delta rows
-        // have the donor store's layout.
-        const long rows_c = long(d->P) * sh.num_layers * sh.num_kv_heads * d->Tp;
-        const long rows_d = d->Dst ? rows_c * d->Dst : rows_c;
-        const DeltaLayout dl = delta_layout(d);
-        const void* xk = d->delta_on ? static_cast<const void*>(d->delta + dl.k_off) : k_clean;
-        const void* xv = d->delta_on ? static_cast<const void*>(d->delta + dl.v_off) : v_clean;
-        const void* ptrs[6] = {k_clean, v_clean, d->Dst ? k_donor : k_clean, d->Dst ? v_donor : v_clean, xk, xv};
-        const long rows[6] = {rows_c, rows_c, rows_d, rows_d, d->delta_on ? rows_d : rows_c, d->delta_on ? rows_d : rows_c};
-        const int box = splice::prefix_tc_box_rows(sh.head_dim);
-        for (int i = 0; i < 6; ++i) {
-            if (d->map_ptr[i] == ptrs[i]) continue;
-            if (splice::make_kv_tensor_map(d->maps[i], ptrs[i], rows[i], sh.head_dim, box) != 0)
-                return fail(SPLICE_ECUDA, "cuTensorMapEncodeTiled failed for store %d", i);
-            d->map_ptr[i] = ptrs[i];
-        }
-        const bool overlap = gs_launched && !d->profiling;
-        e = timed_launch(d, 1, stream, [&] {
-            return splice::launch_prefix_tc(p, d->maps, bounds, tc_keys, stream, overlap);
-        });
-        if (e != cudaSuccess) return cuda_fail(e, "prompt-span tensor-core pass launch");
-    }
-    const bool merge_overlap = prefix_launched && !d->profiling;
-    e = timed_launch(d, 3, stream, [&] { return splice::launch_merge(p, stream, merge_overlap); });
-    if (e != cudaSuccess) return cuda_fail(e, "merge launch");
-    return SPLICE_OK;
+splice_status spliced_decode_step(splice_desc* d, int layer, int step, const splice_bf16* q,
+                                  const splice_bf16* k_new, const splice_bf16* v_new,
+                                  const splice_bf16* k_clean, const splice_bf16* v_clean,
+                                  const splice_bf16* k_donor, const splice_bf16* v_donor, splice_bf16* k_suffix,
+                                  splice_bf16* v_suffix, float* out, void* workspace, size_t workspace_bytes,
+                                  void* stream) {
+    if (d && (step < 1 || step > d->T))
+        return fail(SPLICE_EINVAL, "spliced_decode_step: step %d not in [1, %d]", step, d->T);
+    if (!k_new || !v_new) return fail(SPLICE_EINVAL, "spliced_decode_step: NULL k_new or v_new");
+    return attn_common(d, layer, step, q, k_new, v_new, k_clean, v_clean, k_donor, v_donor, k_suffix, v_suffix,
+                       out, workspace, workspace_bytes, stream, "spliced_decode_step");
 }
 
 size_t splice_delta_bytes(const splice_desc* d) { return d ? delta_layout(d).total : 0; }
@@ -603,7 +627,6 @@ splice_status splice_delta_build(splice_desc* d, const splice_bf16* k_clean, con
     if (e != cudaSuccess) return cuda_fail(e, "earlier CUDA error");
     const splice_model_shape& sh = d->shape;
     char* b = static_cast<char*>(delta);
-    d->append_layer = d->append_step = -1;
     e = cudaError_t(splice::launch_delta_build(
         k_clean, v_clean, k_donor, v_donor, reinterpret_cast<uint32_t*>(b + dl.mask_off),
         reinterpret_cast<int32_t*>(b + dl.count_off), reinterpret_cast<uint16_t*>(b + dl.k_off),
@@ -761,9 +784,17 @@ splice_status splice_debug_wait_timeout(splice_desc* d, unsigned limit_us, void*
     if (limit_us == 0 || limit_us > 1000000u) return fail(SPLICE_EINVAL, "limit_us %u not in [1, 1000000]", limit_us);
     DeviceGuard g(d->device);
     if (g.err != cudaSuccess) return cuda_fail(g.err, "cudaSetDevice");
-    d->append_layer = d->append_step = -1;
     cudaError_t e = cudaError_t(splice::launch_wait_timeout(d->d_err, 1000ull * limit_us, stream));
     if (e != cudaSuccess) return cuda_fail(e, "wait-timeout launch");
+    return SPLICE_OK;
+}
+
+splice_status splice_debug_late_copy(void* dst, const void* src, size_t bytes, unsigned delay_us, void* stream) {
+    if (!dst || !src || !aligned16(dst) || !aligned16(src) || bytes % 16 != 0)
+        return fail(SPLICE_EINVAL, "splice_debug_late_copy: NULL or misaligned buffer, or bytes not a multiple of 16");
+    if (delay_us > 1000000u) return fail(SPLICE_EINVAL, "delay_us %u above 1000000", delay_us);
+    cudaError_t e = cudaError_t(splice::launch_late_copy(dst, src, bytes, 1000ull * delay_us, stream));
+    if (e != cudaSuccess) return cuda_fail(e, "late-copy launch");
     return SPLICE_OK;
 }
 

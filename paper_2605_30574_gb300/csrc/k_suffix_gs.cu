@@ -34,7 +34,7 @@ namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
 constexpr float kTau = 8.0f;
-constexpr unsigned kErrWaitGs = 0x10;
+constexpr unsigned kErrWaitGs = 0x10, kErrWaitGsDrain = 0x80;
 
 __device__ __forceinline__ float ex2(float x) {
     float y;
@@ -125,20 +125,15 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
     extern __shared__ __align__(128) uint8_t smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     // Launched as a programmatic dependent of whatever precedes it on the
-    // stream, this grid may start before that grid has finished.  Where the
-    // host knows the preceding grid is the append of this very layer and
-    // step (P.dep_late), which writes generated-span entry step - 1 and
-    // nothing else this pass reads, the wait for it comes only before the
-    // first copy of a block that holds that entry, and the blocks before it
-    // stream in the meantime; otherwise it comes first.  A no-op for a plain
-    // launch.  The prompt-span pass queued behind this grid reads nothing it
-    // writes: let it start as soon as SMs free up.
+    // stream, this grid may start before that grid has finished: wait for it
+    // (its writes visible) before reading or writing anything.  A no-op for a
+    // plain launch.  Only then may the prompt-span pass queued behind this
+    // grid start: it reads the queries and the prompt stores without a wait
+    // of its own, so its start must imply that everything before this grid
+    // on the stream is complete.  It reads nothing this grid writes, so it
+    // may take the SMs this grid's last CTAs leave idle.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-    bool dep_done = false;
-    if (!P.dep_late) {
-        asm volatile("griddepcontrol.wait;" ::: "memory");
-        dep_done = true;
-    }
     uint8_t* ws = smem + warp * C::PER_WARP;
     const uint32_t wbase = tc::smem_u32(ws);
     const uint32_t bar0 = wbase + C::OFF_BAR;
@@ -173,17 +168,18 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
         if (!iss_ok) return;
         const int stg = issued & 1;
         const int j = iss.k0 + iss_b * 16;
-        const int nk = min(16, iss.k1 - j);
+        int nk = min(16, iss.k1 - j);
+        // fused append: entry step - 1 (the block's last row) is not in the
+        // store yet; the consumer writes that row of the stage from registers
+        if (P.fuse_append && j + nk == P.s_hi) --nk;
         const uint32_t bytes = uint32_t(nk) * C::ROW;
-        if (!dep_done && j + nk >= P.s_hi) {
-            asm volatile("griddepcontrol.wait;" ::: "memory");
-            dep_done = true;
-        }
         if (lane == 0) {
             const uint32_t dst = wbase + stg * C::STAGE;
             tc::mbar_arrive_expect_tx(bar0 + 8 * stg, 2 * bytes);
-            bulk_copy(dst, iss.k + size_t(j) * D, bytes, bar0 + 8 * stg, pol);
-            bulk_copy(dst + C::BK * C::ROW, iss.v + size_t(j) * D, bytes, bar0 + 8 * stg, pol);
+            if (bytes) {
+                bulk_copy(dst, iss.k + size_t(j) * D, bytes, bar0 + 8 * stg, pol);
+                bulk_copy(dst + C::BK * C::ROW, iss.v + size_t(j) * D, bytes, bar0 + 8 * stg, pol);
+            }
         }
         ++issued;
         if (++iss_b >= iss.nblk) {
@@ -227,6 +223,23 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
             for (int i = 0; i < 8; ++i) o2[g][i] = make_float2(0.f, 0.f);
         }
         float m_mine = -INFINITY, l_mine = 0.f;
+        // fused append: this item's split ends at the step's own entry (step
+        // - 1), which comes from the new K/V rows, loaded now (lanes take
+        // 16-byte chunks: the K row's D / 8, then the V row's)
+        constexpr int NCH = D / 4;                       // 16-byte chunks of the K and V rows
+        constexpr int CPL = NCH >= 32 ? NCH / 32 : 1;    // chunks per lane
+        const bool tail = P.fuse_append && it.k1 == P.s_hi && it.nblk > 0;
+        uint4 nkv[CPL];
+        if (tail) {
+            const size_t rowc = (size_t(it.s) * P.Hkv + it.h) * (D / 8);
+#pragma unroll
+            for (int i = 0; i < CPL; ++i) {
+                const int c = lane + 32 * i;
+                if (c < NCH)
+                    nkv[i] = c < D / 8 ? reinterpret_cast<const uint4*>(P.kn)[rowc + c]
+                                       : reinterpret_cast<const uint4*>(P.vn)[rowc + c - D / 8];
+            }
+        }
 
         for (int b = 0; b < it.nblk; ++b) {
             const int stg = consumed & 1;
@@ -235,9 +248,27 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
                 ok = false;
                 break;
             }
-            const uint8_t* kst = ws + stg * C::STAGE;
-            const uint8_t* vst = kst + C::BK * C::ROW;
+            uint8_t* kst = ws + stg * C::STAGE;
+            uint8_t* vst = kst + C::BK * C::ROW;
             const int jb = it.k0 + b * 16;
+            if (tail && b == it.nblk - 1) {
+                // the step's own entry: its row of the stage from registers,
+                // and (once per (sequence, kv head)) into the store
+                const int rj = P.s_hi - 1 - jb;
+                const size_t ent = ((size_t(it.s) * P.N + P.layer) * P.Hkv + it.h) * size_t(P.T) + (P.s_hi - 1);
+#pragma unroll
+                for (int i = 0; i < CPL; ++i) {
+                    const int c = lane + 32 * i;
+                    if (c < NCH) {
+                        const bool isk = c < D / 8;
+                        const int cc = isk ? c : c - D / 8;
+                        *reinterpret_cast<uint4*>((isk ? kst : vst) + rj * C::ROW + cc * 16) = nkv[i];
+                        if (it.rc == 0)
+                            reinterpret_cast<uint4*>(isk ? P.ks_w : P.vs_w)[ent * (D / 8) + cc] = nkv[i];
+                    }
+                }
+                __syncwarp();
+            }
 
             // ---- partial q . k over this lane's 16 dims ----
             float dot[C::NV];
@@ -400,13 +431,15 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
             }
         }
     }
-    // This grid's completion implies the preceding grid's for whatever is
-    // queued after it.
-    if (!dep_done) asm volatile("griddepcontrol.wait;" ::: "memory");
-    // Copies still in flight (only after an abort) must land before exit.
+    // Copies still in flight (only after an abort: at most the two of the
+    // ring) must land before the warp's shared memory is given up.  A bulk
+    // copy from global memory waits on nothing else on the GPU, so it lands;
+    // the long bound only keeps a broken memory system from holding the CTA
+    // forever, and a drain that runs out records its own error bit.
     for (; consumed < issued; ++consumed) {
         volatile int no_abort = 0;
-        tc::mbar_wait(bar0 + 8 * (consumed & 1), uint32_t(consumed >> 1) & 1u, &no_abort, P.err, kErrWaitGs);
+        tc::mbar_wait(bar0 + 8 * (consumed & 1), uint32_t(consumed >> 1) & 1u, &no_abort, P.err, kErrWaitGsDrain,
+                      10000000000ull);
     }
 }
 

@@ -81,6 +81,13 @@ struct AttnParams {
     const uint16_t* vd;
     const uint16_t* ks;
     const uint16_t* vs;
+    // fused append (fuse_append != 0): this step's entries [B][Hkv][D], written
+    // by the generated-span pass to entry step - 1 of ks_w / vs_w (the same
+    // store as ks / vs) and read from registers instead of from the store
+    const uint16_t* kn;
+    const uint16_t* vn;
+    uint16_t* ks_w;
+    uint16_t* vs_w;
     float* out;
     float2* ws_ml;          // [kMaxSplits][B * Hq] (m in log2 units, l)
     float* ws_o;            // [kMaxSplits][B * Hq][D]
@@ -105,7 +112,7 @@ struct AttnParams {
     int nsp, nss;                 // splits of the prompt span / generated span
     int nsd;                      // splits of the delta rows (delta mode)
     int delta_on, delta_w32;
-    int dep_late;                 // the preceding grid is this layer and step's append (see gs_kernel)
+    int fuse_append;              // the generated-span pass also appends entry step - 1 (see kn, vn)
     int p_chunk, s_chunk;         // keys per split
     int n_tiles;
     int n_span_tiles;             // tiles [0, n_span_tiles) read stored spans, the rest delta rows
@@ -115,16 +122,26 @@ struct AttnParams {
 // Records the one-line reason splice_last_error() reports on this thread.
 void set_last_error(const char* msg);
 
+// The device a (device) descriptor was created on and launches on; -1 for a
+// host-only descriptor or NULL.
+int desc_device(const splice_desc* d);
+
 // Launchers (return the cudaError_t of the launch as int).
 int launch_append(const uint16_t* kn, const uint16_t* vn, uint16_t* ks, uint16_t* vs, int B,
                   int N, int Hkv, int D, int T, int layer, int step, void* stream);
 // overlap_previous: launched as a programmatic dependent of the preceding
-// work on the stream (the kernel waits for it before reading anything).
+// work on the stream (the kernel waits for it before reading or writing
+// anything, and lets its own dependents launch only after that wait).
 int launch_generated_span(const AttnParams& p, void* stream, bool overlap_previous);
 int generated_span_resident_warps(int d);
 // overlap_previous: the launch directly follows the prompt-span pass on the
 // same stream (programmatic dependent launch; the kernel waits for it).
 int launch_merge(const AttnParams& p, void* stream, bool overlap_previous);
+
+// A copy of `bytes` (a multiple of 16) from src to dst by a kernel that lets
+// its programmatic dependents launch at its start and copies only after
+// delay_ns.
+int launch_late_copy(void* dst, const void* src, size_t bytes, unsigned long long delay_ns, void* stream);
 
 // One-thread kernel whose mbarrier wait runs out after limit_ns.
 int launch_wait_timeout(unsigned* err, unsigned long long limit_ns, void* stream);

@@ -53,8 +53,11 @@ SIGNATURES = {
     "suffix_kv_append": (_c_int, [_vp, _c_int, _c_int, _vp, _vp, _vp, _vp, _vp]),
     "spliced_decode_attn": (_c_int, [_vp, _c_int, _c_int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
                                      _vp, _c_size, _vp]),
+    "spliced_decode_step": (_c_int, [_vp, _c_int, _c_int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                     _vp, _c_size, _vp]),
     "spliced_decode_attn_static": (_c_int, [_vp, _c_int, _c_int, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
                                             _vp]),
+    "splice_static_scratch_bytes": (_c_size, []),
     "splice_debug_source_map": (_c_int, [_vp, _c_int, _c_int, ctypes.POINTER(ctypes.c_uint8)]),
     "splice_plan_stats": (_c_int, [_vp, _c_int, _c_int, ctypes.POINTER(_c_int), ctypes.POINTER(_c_int),
                                    ctypes.POINTER(_c_int), ctypes.POINTER(_c_int)]),
@@ -67,6 +70,7 @@ SIGNATURES = {
                                         ctypes.POINTER(_c_int)]),
     "splice_check_device_error": (_c_int, [_vp]),
     "splice_debug_wait_timeout": (_c_int, [_vp, ctypes.c_uint, _vp]),
+    "splice_debug_late_copy": (_c_int, [_vp, _vp, _c_size, ctypes.c_uint, _vp]),
     "splice_kernel_launches": (ctypes.c_longlong, [_vp]),
     "splice_profile_enable": (_c_int, [_vp, _c_int]),
     "splice_profile_read": (_c_int, [_vp, ctypes.POINTER(ctypes.c_longlong), ctypes.POINTER(ctypes.c_double)]),
@@ -199,7 +203,21 @@ def spliced_decode_attn(desc: Desc, layer, step, q, k_clean, v_clean, k_donor, v
            "spliced_decode_attn")
 
 
-STATIC_SCRATCH_BYTES = 64 << 20
+def spliced_decode_step(desc: Desc, layer, step, q, k_new, v_new, k_clean, v_clean, k_donor, v_donor, k_suffix,
+                        v_suffix, out, workspace, workspace_bytes=None, stream=None):
+    """suffix_kv_append + spliced_decode_attn in one call (the append runs
+    inside the generated-span pass)."""
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    _check(lib().spliced_decode_step(desc.handle, layer, step, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_clean),
+                                     _ptr(v_clean), _ptr(k_donor), _ptr(v_donor), _ptr(k_suffix), _ptr(v_suffix),
+                                     _ptr(out), _ptr(workspace), workspace_bytes, _stream(stream)),
+           "spliced_decode_step")
+
+
+def splice_static_scratch_bytes() -> int:
+    """Size of the no-allocation entry point's static scratch, as the library was built."""
+    return int(lib().splice_static_scratch_bytes())
 
 
 def spliced_decode_attn_static(desc: Desc, layer, step, q, k_clean, v_clean, k_donor, v_donor, k_suffix,
@@ -269,6 +287,13 @@ def splice_debug_plan_rows(desc: Desc, layer, step) -> list:
 
 def splice_debug_wait_timeout(desc: Desc, limit_us: int, stream=None):
     _check(lib().splice_debug_wait_timeout(desc.handle, limit_us, _stream(stream)), "splice_debug_wait_timeout")
+
+
+def splice_debug_late_copy(dst, src, delay_us: int, stream=None):
+    """dst <- src (same size) by a kernel that lets dependents launch at once and copies after delay_us."""
+    nbytes = src.numel() * src.element_size()
+    _check(lib().splice_debug_late_copy(_ptr(dst), _ptr(src), nbytes, int(delay_us), _stream(stream)),
+           "splice_debug_late_copy")
 
 
 def splice_check_device_error(desc: Desc):

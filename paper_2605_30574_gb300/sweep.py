@@ -86,6 +86,13 @@ class SweepBatch:
                               self.k_donor, self.v_donor, self.k_suffix, self.v_suffix,
                               self.out if out is None else out, self.ws, stream=stream)
 
+    def step(self, layer: int, step: int, q=None, k_new=None, v_new=None, out=None, stream=None):
+        """The fused call: append this step's K/V and attend (step >= 1)."""
+        S.spliced_decode_step(self.desc, layer, step, self.q if q is None else q,
+                              self.k_new if k_new is None else k_new, self.v_new if v_new is None else v_new,
+                              self.k_clean, self.v_clean, self.k_donor, self.v_donor, self.k_suffix, self.v_suffix,
+                              self.out if out is None else out, self.ws, stream=stream)
+
     def run(self, layer: int, step: int):
         """Generate inputs, append (step >= 1) and attend; returns self.out."""
         self.gen_inputs(layer, step)

@@ -1,6 +1,8 @@
 """The bench's algorithmic-byte count, on host descriptors (no GPU): one
-read of every distinct (prompt, source) span a layer-step touches plus the
-queries; in delta-donor mode a reader of an encoded slot adds its prompt's
+read of every distinct (prompt, source) span a layer-step touches, every
+sequence's visible generated entries, each query once, the outputs and the
+appended entries (moved by the generated-span pass in the fused call); in
+delta-donor mode a reader of an encoded slot adds its prompt's
 clean span (shared) and the slot's encoded rows instead of the donor span."""
 from types import SimpleNamespace
 
@@ -34,14 +36,19 @@ def test_bytes_by_hand():
     q = 4 * 64 * 2
     b = bench.algorithmic_bytes(sb, 0, 1)
     # spans: (0, SAME_ALGO), (0, clean), (1, clean), (1, BLANK); 4 readers
-    assert b["prompt_span_pass"] == 4 * 100 * kv_pos + 4 * q
+    assert b["prompt_span_pass"] == 4 * 100 * kv_pos
     assert b["generated_span_pass"] == 5 * 1 * kv_pos + 5 * q
     assert b["merge"] == 5 * 4 * 64 * 4 and b["append"] == 5 * 2 * 64 * 8
+    # the total is the per-step formula: spans + generated entries + B Hq d (2 q + 4 out) + appends
+    assert sum(b.values()) == 4 * 100 * kv_pos + 5 * 1 * kv_pos + 5 * 4 * 64 * (2 + 4) + 5 * 2 * 64 * 8
+    bf = bench.algorithmic_bytes(sb, 0, 1, fused=True)
+    assert bf["append"] == 0 and bf["generated_span_pass"] == b["generated_span_pass"] + b["append"]
+    assert sum(bf.values()) == sum(b.values())
     # delta mode for SAME_ALGO (stored slot 0): prompt 0's reader adds the
     # clean span it already shares and 7 + 5 encoded rows (two kv heads)
     counts = np.zeros((2, 2, 1, 2), np.int64)
     counts[0, 0, 0] = (7, 5)
     counts[1, 0, 0] = (40, 40)                 # prompt 1 has no SAME_ALGO reader at this step
     bd = bench.algorithmic_bytes(sb, 0, 1, ([True, False, False], counts))
-    assert bd["prompt_span_pass"] == 3 * 100 * kv_pos + (7 + 5) * 64 * 4 + 4 * q
+    assert bd["prompt_span_pass"] == 3 * 100 * kv_pos + (7 + 5) * 64 * 4
     assert bd["generated_span_pass"] == b["generated_span_pass"]

@@ -59,6 +59,15 @@ def test_decode_step_graph_replays_bit_exact(step):
         torch.cuda.synchronize()
         for l in range(N):
             assert torch.equal(outs_graph[l], outs_eager[l]), f"layer {l}"
+    # and the replayed step against the fp64 oracle on sampled rows of every layer
+    import oracle
+    from parity_util import CachedInputs, assert_close
+    inp = CachedInputs(wl)
+    for l in range(N):
+        g_l = outs_graph[l].cpu().numpy()
+        for s in range(0, sb.B, 9):
+            ref = oracle.decode_attn(wl, inp, sb.s0 + s, sb.seqs[s], l, step)
+            assert_close(g_l[s], ref, f"graph layer {l} s={s} step={step}")
     from paper_2605_30574_gb300 import splice as S
     S.splice_check_device_error(sb.desc)
     sb.close()
@@ -110,3 +119,43 @@ def test_decode_step_graph_in_delta_mode():
         assert_close(outs_graph[l][torch.tensor(rows, device="cuda")].cpu().numpy(), ref, f"delta graph l={l}")
     S.splice_check_device_error(sb.desc)
     sb.close()
+
+
+def test_fused_decode_step_graph_replays_bit_exact():
+    """A whole decode step through the fused call (every layer's append done
+    inside its generated-span pass) captured into one graph: replays equal
+    the unfused calls issued one by one, outputs and generated-span store."""
+    wl = ladder_slice()
+    a = SweepBatch(wl, 0)
+    b = SweepBatch(wl, 0)
+    N, step = wl.num_layers, 300
+    qs, kns, vns = [], [], []
+    for l in range(N):
+        a.gen_inputs(l, step)
+        qs.append(a.q.clone())
+        kns.append(a.k_new.clone())
+        vns.append(a.v_new.clone())
+    outs_eager = [torch.empty_like(a.out) for _ in range(N)]
+    for l in range(N):
+        a.append(l, step, kns[l], vns[l])
+        a.attn(l, step, q=qs[l], out=outs_eager[l])
+    torch.cuda.synchronize()
+    outs_graph = [torch.full_like(b.out, float("nan")) for _ in range(N)]
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for l in range(N):
+            b.step(l, step, q=qs[l], k_new=kns[l], v_new=vns[l], out=outs_graph[l])
+    for _ in range(2):
+        for o in outs_graph:
+            o.fill_(float("nan"))
+        b.k_suffix[:, :, :, step - 1].zero_()
+        b.v_suffix[:, :, :, step - 1].zero_()
+        g.replay()
+        torch.cuda.synchronize()
+        for l in range(N):
+            assert torch.equal(outs_graph[l], outs_eager[l]), f"layer {l}"
+        assert torch.equal(b.k_suffix, a.k_suffix) and torch.equal(b.v_suffix, a.v_suffix)
+    from paper_2605_30574_gb300 import splice as S
+    S.splice_check_device_error(b.desc)
+    a.close()
+    b.close()

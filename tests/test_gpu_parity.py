@@ -239,6 +239,53 @@ def test_full_size_sampled(name):
     print(name, "points", len(got), "worst abs/rel", worst)
 
 
+@pytest.mark.parametrize("name", ["qwen3-8b-ladder"])
+def test_ladder_first_and_last_prompt_every_cell(name):
+    """The sampling plan for the donor-noise ladder: every cell of the first
+    and the last prompt -- prompt 0 in batch 0, prompt P - 1 in the last,
+    ragged batch of 128 sequences -- at steps {1, W - 1, W, W + 1, T / 2, T}
+    and layers {0, L - 1, L, N - 1} around the cell's own onset and cutoff,
+    in the launch configuration the bench times (whole batches)."""
+    from oracle_pool import oracle_outputs
+    wl = WL.get(name)
+    N, T = wl.num_layers, wl.max_steps
+    seqs = wl.sequences()
+    units = []
+    for s, q in enumerate(seqs):
+        if q.prompt not in (0, wl.num_prompts - 1):
+            continue
+        layers = {x for x in (0, q.L - 1, q.L, N - 1) if 0 <= x < N}
+        steps = {x for x in (1, q.W - 1, q.W, q.W + 1, T // 2, T) if 1 <= x <= T}
+        units += [(s, l, t) for l in layers for t in steps]
+    batches = sorted({s // wl.batch for s, _, _ in units})
+    assert batches == [0, wl.num_batches() - 1]
+    assert wl.batch_range(batches[-1])[1] - wl.batch_range(batches[-1])[0] == 128
+    got = {}
+    for b in batches:
+        torch.cuda.empty_cache()
+        sb = SweepBatch(wl, b)
+        lo = sb.s0
+        by_lt = {}
+        for s, l, t in units:
+            if lo <= s < lo + sb.B:
+                by_lt.setdefault((l, t), []).append(s)
+        for (l, t), ss in sorted(by_lt.items(), key=lambda kv: (kv[0][1], kv[0][0])):
+            out = sb.run(l, t)
+            rows = out[torch.tensor([s - lo for s in ss], device="cuda")].cpu().numpy()
+            for s, r in zip(ss, rows):
+                got[(s, l, t)] = r
+        S.splice_check_device_error(sb.desc)
+        sb.close()
+        del sb
+    torch.cuda.empty_cache()
+    ref = oracle_outputs(name, units)
+    worst = (0.0, 0.0)
+    for u in sorted(got):
+        a, r = assert_close(got[u], ref[u], f"{name} s={u[0]} l={u[1]} t={u[2]}")
+        worst = (max(worst[0], a), max(worst[1], r))
+    print(name, "units", len(got), "worst abs/rel", worst)
+
+
 # --------------------------------------------------------------------------
 # softmax scale: sign and zero
 # --------------------------------------------------------------------------
