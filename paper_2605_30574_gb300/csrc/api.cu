@@ -26,6 +26,7 @@ struct splice_desc {
     std::vector<splice_seq> seqs;
     Plan plan;
     int device = -1;
+    int sms = 0;                        // multiprocessors of the device
     // Device tables, one allocation.
     char* dev = nullptr;
     std::vector<char> staging;          // host image of `dev`, kept for the async upload
@@ -40,7 +41,7 @@ struct splice_desc {
     int32_t* d_group_mask = nullptr;
     int32_t* d_slot_delta = nullptr;
     unsigned* d_err = nullptr;
-    unsigned* d_sched = nullptr;   // [2] prompt-span work counter, finished-CTA count (zero between launches)
+    unsigned* d_sched = nullptr;   // [4] work counter and finished-CTA count of each pass (zero between launches)
     // Measurement: launch counter and optional per-launch event timing.
     long long launches = 0;
     bool profiling = false;
@@ -190,7 +191,7 @@ splice_status upload_tables(splice_desc* d, void* stream) {
     }
     for (int k = 0; k < d->Dslots; ++k) slot_delta[k] = d->slot_delta[k] ? 1 : 0;
     const unsigned zero = 0;
-    const unsigned sched_zero[2] = {0, 0};
+    const unsigned sched_zero[4] = {0, 0, 0, 0};
     Part parts[] = {
         {pl.src.data(), pl.src.size(), 0},
         {seq_prompt.data(), seq_prompt.size() * 4, 0},
@@ -439,22 +440,33 @@ splice_status attn_common(splice_desc* d, int layer, int step, const splice_bf16
     p.s_chunk = p.nss ? (s_vis + p.nss - 1) / p.nss : 0;
     p.scale_log2 = sh.sm_scale * 1.4426950408889634f;
 
-    // The two passes read disjoint inputs and write disjoint partial slots.
-    // The generated-span pass goes first; the prompt-span pass is queued
-    // right behind it as a programmatic dependent launch, so its CTAs fill
-    // the SMs the generated-span pass's last CTAs leave idle, and it waits
-    // for that pass before it exits.  With per-launch timing on, the events
-    // between the launches serialise them instead.  (A fused call always has
-    // a generated span: step >= 1.)
-    const bool gs_launched = p.nss > 0;
-    if (gs_launched) {
-        e = timed_launch(d, 2, stream, [&] { return splice::launch_generated_span(p, stream, !d->profiling); });
-        if (e != cudaSuccess) return cuda_fail(e, "generated-span partials launch");
-    }
+    // The two passes read disjoint inputs and write disjoint partial slots,
+    // and run as programmatic dependent launches: the call's first pass
+    // waits for whatever precedes it on the stream before it reads anything,
+    // then lets the second pass launch; the second pass's CTAs take the SMs
+    // the first pass's CTAs leave, and it waits for the first pass before it
+    // exits; the merge is queued behind the second pass.  So the first pass's
+    // tail is filled and the second pass's is not.  The generated-span pass
+    // goes first when the prompt-span pass holds at least one full split
+    // (kPrefixSplitKeys keys) per SM: then the prompt-span pass's items fill
+    // the generated-span pass's tail.  A smaller prompt-span pass goes first:
+    // its short run and its tail (part of the SMs idle while its last items
+    // finish) are filled by the generated-span pass's run-time claimed
+    // units.  With per-launch timing on, the events between the launches
+    // serialise everything.
+    const bool gs_work = p.nss > 0;
     const long prefix_items = long(p.n_span_tiles) * sh.num_kv_heads * p.nsp +
                               long(p.n_tiles - p.n_span_tiles) * sh.num_kv_heads * p.nsd;
     const bool prefix_launched = p.nsp > 0 && prefix_items > 0;
-    if (prefix_launched) {
+    const int box = splice::prefix_tc_box_rows(sh.head_dim);
+    const long prefix_keys =
+        (long(p.n_span_tiles) * ((p_vis + box - 1) / box) +
+         long(p.n_tiles - p.n_span_tiles) * (p.nsd ? (d->delta_max + box - 1) / box : 0)) *
+        sh.num_kv_heads * box;
+    const bool prefix_first = prefix_launched && prefix_keys < long(d->sms) * splice::kPrefixSplitKeys;
+    p.gs_after_prefix = gs_work && prefix_launched && prefix_first && !d->profiling ? 1 : 0;
+    p.prefix_after_gs = gs_work && prefix_launched && !prefix_first && !d->profiling ? 1 : 0;
+    auto launch_prefix = [&]() -> splice_status {
         // Tensor maps over the stores viewed as [rows][d]; the delta rows
         // have the donor store's layout.
         const long rows_c = long(d->P) * sh.num_layers * sh.num_kv_heads * d->Tp;
@@ -465,20 +477,37 @@ splice_status attn_common(splice_desc* d, int layer, int step, const splice_bf16
         const void* mp[6] = {k_clean, v_clean, d->Dst ? k_donor : k_clean, d->Dst ? v_donor : v_clean, xk, xv};
         const long mrows[6] = {rows_c, rows_c, rows_d, rows_d, d->delta_on ? rows_d : rows_c,
                                d->delta_on ? rows_d : rows_c};
-        const int box = splice::prefix_tc_box_rows(sh.head_dim);
         for (int i = 0; i < 6; ++i) {
             if (d->map_ptr[i] == mp[i]) continue;
             if (splice::make_kv_tensor_map(d->maps[i], mp[i], mrows[i], sh.head_dim, box) != 0)
                 return fail(SPLICE_ECUDA, "cuTensorMapEncodeTiled failed for store %d", i);
             d->map_ptr[i] = mp[i];
         }
-        const bool overlap = gs_launched && !d->profiling;
-        e = timed_launch(d, 1, stream, [&] {
-            return splice::launch_prefix_tc(p, d->maps, bounds, tc_keys, stream, overlap);
+        const cudaError_t le = timed_launch(d, 1, stream, [&] {
+            return splice::launch_prefix_tc(p, d->maps, bounds, tc_keys, stream, !d->profiling);
         });
-        if (e != cudaSuccess) return cuda_fail(e, "prompt-span tensor-core pass launch");
+        if (le != cudaSuccess) return cuda_fail(le, "prompt-span tensor-core pass launch");
+        return SPLICE_OK;
+    };
+    auto launch_gs = [&]() -> splice_status {
+        const cudaError_t le =
+            timed_launch(d, 2, stream, [&] { return splice::launch_generated_span(p, stream, !d->profiling); });
+        if (le != cudaSuccess) return cuda_fail(le, "generated-span partials launch");
+        return SPLICE_OK;
+    };
+    if (prefix_launched && prefix_first) {
+        const splice_status st = launch_prefix();
+        if (st != SPLICE_OK) return st;
     }
-    const bool merge_overlap = prefix_launched && !d->profiling;
+    if (gs_work) {
+        const splice_status st = launch_gs();
+        if (st != SPLICE_OK) return st;
+    }
+    if (prefix_launched && !prefix_first) {
+        const splice_status st = launch_prefix();
+        if (st != SPLICE_OK) return st;
+    }
+    const bool merge_overlap = (prefix_launched || gs_work) && !d->profiling;
     e = timed_launch(d, 3, stream, [&] { return splice::launch_merge(p, stream, merge_overlap); });
     if (e != cudaSuccess) return cuda_fail(e, "merge launch");
     return SPLICE_OK;
@@ -526,6 +555,11 @@ splice_status splice_desc_create(const splice_model_shape* sh, int P, int Tp, in
     if (e != cudaSuccess) {
         delete d;
         return cuda_fail(e, "cudaGetDevice");
+    }
+    e = cudaDeviceGetAttribute(&d->sms, cudaDevAttrMultiProcessorCount, d->device);
+    if (e != cudaSuccess) {
+        delete d;
+        return cuda_fail(e, "cudaDeviceGetAttribute");
     }
     st = upload_tables(d, stream);
     if (st != SPLICE_OK) {

@@ -64,9 +64,12 @@ constexpr float kTau = 8.0f;        // lazy rescale threshold, log2 units
 
 constexpr unsigned kErrWaitProducer = 0x1, kErrWaitMma = 0x2, kErrWaitSoftmax = 0x4, kErrWaitDrain = 0x8,
                    kErrWaitQ = 0x20, kErrWaitItem = 0x40;
-// Work items reach the CTA's roles through a ring of item numbers in smem.
+// Work items reach the CTA's roles through a ring in smem: the producer
+// posts every item decoded (tile, kv head, split, span), so no other role
+// reads the tile tables.
 constexpr int kItemRing = 8;
 constexpr int kItemTakers = 12;     // Q K^T warp, P V warp, Q gather warp, 8 softmax warps, the V cursor
+constexpr uint32_t kRingEntryBytes = 64;
 
 __device__ __forceinline__ float ex2(float x) {
     float y;
@@ -93,6 +96,16 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&v)[16
         : "memory");
 }
 
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&v)[8]) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"r"(taddr),
+                 "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
+                 : "memory");
+}
+
+// One segment's P (bf16 pairs), by segment size.
+__device__ __forceinline__ void store_p(uint32_t taddr, const uint32_t (&v)[16]) { tmem_st16(taddr, v); }
+__device__ __forceinline__ void store_p(uint32_t taddr, const uint32_t (&v)[8]) { tmem_st8(taddr, v); }
+
 template <int D>
 struct Cfg {
     static constexpr int BN = D == 256 ? 64 : 128;          // keys per K/V block
@@ -117,7 +130,8 @@ struct Cfg {
     static constexpr uint32_t OFF_X = OFF_V + VST * KV_BYTES;
     static constexpr uint32_t X_BYTES = 2 * (2 * 2 * kRows) * 4;
     static constexpr uint32_t OFF_BAR = OFF_X + X_BYTES;
-    static constexpr uint32_t SMEM = OFF_BAR + 1024 + 1024;   // + barriers, + alignment slack
+    static constexpr uint32_t OFF_RING = OFF_BAR + 1024;    // [kItemRing] posted work items
+    static constexpr uint32_t SMEM = OFF_RING + kItemRing * kRingEntryBytes + 1024;   // + alignment slack
     static_assert(NSLOT >= 2 && COL_O + D <= kTmemCols, "TMEM budget");
     static_assert(SMEM <= 227 * 1024, "shared memory budget");
     static_assert(KPT % 32 == 0 && OCH % 32 == 0 && VST >= 2, "TMEM access granularity, ring depth");
@@ -161,15 +175,18 @@ struct TcParams {
 // launch ends on short items).  Items over stored spans come first, then
 // the items over delta rows (their own split count).
 struct ItemInfo {
+    int item;           // the item's number; -1 after the CTA's last item, -2 when a wait gave up
     int h, split, first, nseq, k0, k1, nblk, prompt;
     int store;          // 0 clean, 1 donor, 2 delta rows
     bool masked;        // a clean span in delta mode: rows may drop encoded positions
     long span_row;      // first row of the span in the store's 2D view
 };
+static_assert(sizeof(ItemInfo) <= kRingEntryBytes, "item ring entry");
 
 template <int D>
 __device__ __forceinline__ ItemInfo item_info(const AttnParams& P, const TcParams& tp, int item) {
     ItemInfo it;
+    it.item = item;
     int tile, split;
     if (item < tp.n_span_items) {
         tile = item % P.n_span_tiles;
@@ -186,30 +203,22 @@ __device__ __forceinline__ ItemInfo item_info(const AttnParams& P, const TcParam
         split = hs / P.Hkv;
         it.split = P.nsp + split;              // after the span's own partials
     }
+    // one 16-byte record per tile: group, first reader, readers, and the
+    // store kind with the span base index (clean: the prompt; donor or delta
+    // rows: prompt * stored slots + stored index)
     const int4 tl = reinterpret_cast<const int4*>(P.tiles)[tile];
     it.first = tl.y;
     it.nseq = tl.z;
-    it.prompt = P.group_prompt[tl.x];
-    const int code = P.group_src[tl.x];
-    long span;
-    if (code & kGroupDelta) {
-        const int st = P.slot_stored[(code & 0xff) - int(SPLICE_SRC_DONOR0)];
-        span = ((long(it.prompt) * P.Dst + st) * P.N + P.layer) * P.Hkv + it.h;
-        it.store = 2;
+    it.store = tl.w & 3;
+    const long base = long(unsigned(tl.w) >> 2);
+    it.prompt = int(base);                     // used by clean spans only
+    const long span = (base * P.N + P.layer) * P.Hkv + it.h;
+    if (it.store == 2) {
         it.masked = false;
         it.k0 = split * tp.delta_keys;
         it.k1 = min(P.dcount[span], it.k0 + tp.delta_keys);
     } else {
-        if (code == int(SPLICE_SRC_CLEAN)) {
-            span = (long(it.prompt) * P.N + P.layer) * P.Hkv + it.h;
-            it.store = 0;
-            it.masked = P.delta_on != 0;
-        } else {
-            const int st = P.slot_stored[code - int(SPLICE_SRC_DONOR0)];
-            span = ((long(it.prompt) * P.Dst + st) * P.N + P.layer) * P.Hkv + it.h;
-            it.store = 1;
-            it.masked = false;
-        }
+        it.masked = it.store == 0 && P.delta_on != 0;
         it.k0 = P.p_lo + tp.sb[split];
         it.k1 = P.p_lo + tp.sb[split + 1];
     }
@@ -235,7 +244,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto bar = [&](int i) { return bar0 + 8u * uint32_t(i); };
     volatile int* s_abort = reinterpret_cast<volatile int*>(smem + C::OFF_BAR + 8 * Bb::COUNT);
     uint32_t* s_tmem = reinterpret_cast<uint32_t*>(smem + C::OFF_BAR + 8 * Bb::COUNT + 8);
-    volatile int* s_items = reinterpret_cast<volatile int*>(smem + C::OFF_BAR + 8 * Bb::COUNT + 16);
+    // The producer posts every item with its decoded fields, so no other
+    // role reads the tile tables.
+    ItemInfo* s_ring = reinterpret_cast<ItemInfo*>(smem + C::OFF_RING);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     if (threadIdx.x == 0) {
@@ -285,18 +296,34 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::tc_fence_before();
     __syncthreads();
     tc::tc_fence_after();
+    // The call's first pass: launched as a programmatic dependent of
+    // whatever precedes it on the stream, this grid may start before that
+    // work has finished, so it waits for it (its writes visible) before
+    // reading anything -- the queries, the work counter, the tables.  Only
+    // then may the generated-span pass queued behind this grid launch: it
+    // reads nothing this grid writes, so its CTAs take the SMs this grid's
+    // CTAs leave, and it waits for this grid before it exits.  (Behind the
+    // generated-span pass instead, that pass has waited before it let this
+    // grid launch; see the end of the kernel.)  No-ops for a plain launch.
+    if (!P.prefix_after_gs) {
+        asm volatile("griddepcontrol.wait;" ::: "memory");
+        asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    }
     const uint32_t tmem = *s_tmem;
-    // Item k of the CTA's stream, for a whole warp: -1 after the last item,
-    // -2 when the wait gave up.
-    auto take_item = [&](int k) -> int {
+    // Item k of the CTA's stream, for a whole warp (item -1 after the last
+    // item, -2 when the wait gave up).
+    auto take_item = [&](int k) -> ItemInfo {
         const int r = k % kItemRing;
+        ItemInfo it;
         if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::IFULL + r), uint32_t(k / kItemRing) & 1u, s_abort, P.err,
-                                                   kErrWaitItem)))
-            return -2;
-        const int item = s_items[r];
+                                                   kErrWaitItem))) {
+            it.item = -2;
+            return it;
+        }
+        it = s_ring[r];
         __syncwarp();
         if (lane == 0) tc::mbar_arrive(bar(Bb::IEMPTY + r));
-        return item;
+        return it;
     };
     // Key block number g of the CTA's stream (counted over all its items)
     // uses S slot g mod NSLOT, for the (g / NSLOT)-th time.
@@ -332,7 +359,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const int r = kpost % kItemRing;
                         if (tc::mbar_test_wait(bar(Bb::IEMPTY + r), (uint32_t(kpost / kItemRing) & 1u) ^ 1u)) {
                             const int item = nxt < tp.n_items ? nxt : -1;
-                            s_items[r] = item;
+                            ItemInfo inf;
+                            inf.item = -1;
+                            if (item >= 0) inf = item_info<D>(P, tp, item);
+                            s_ring[r] = inf;
                             tc::mbar_arrive(bar(Bb::IFULL + r));
                             ++kpost;
                             prog = true;
@@ -340,7 +370,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 k_done = true;
                             } else {
                                 nxt = int(atomicAdd(P.sched, 1u));   // claimed now, needed at the next item
-                                ki = item_info<D>(P, tp, item);
+                                ki = inf;
                                 kj = 0;
                                 k_in = true;
                             }
@@ -366,14 +396,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!v_done) {
                     if (!v_in && vtake < kpost) {
                         const int r = vtake % kItemRing;
-                        const int item = s_items[r];
+                        const ItemInfo inf = s_ring[r];
                         tc::mbar_arrive(bar(Bb::IEMPTY + r));
                         ++vtake;
                         prog = true;
-                        if (item < 0) {
+                        if (inf.item < 0) {
                             v_done = true;
                         } else {
-                            vi = item_info<D>(P, tp, item);
+                            vi = inf;
                             vj = 0;
                             v_in = true;
                         }
@@ -437,12 +467,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool ok = true, committed = false;
         int jg = 0;
         for (int k = 0;; ++k) {
-            const int item = take_item(k);
-            if (item < 0) {
-                ok = item == -1;
+            const ItemInfo it = take_item(k);
+            if (it.item < 0) {
+                ok = it.item == -1;
                 break;
             }
-            const ItemInfo it = item_info<D>(P, tp, item);
             const int qb = C::NQ == 2 ? (k & 1) : 0;
             const uint32_t quse = uint32_t(C::NQ == 2 ? k >> 1 : k);
             const uint32_t q_addr = sbase + C::OFF_Q + qb * C::Q_BYTES;
@@ -492,12 +521,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool ok = true, committed = false;
         int jg = 0;
         for (int k = 0;; ++k) {
-            const int item = take_item(k);
-            if (item < 0) {
-                ok = item == -1;
+            const ItemInfo it = take_item(k);
+            if (it.item < 0) {
+                ok = it.item == -1;
                 break;
             }
-            const ItemInfo it = item_info<D>(P, tp, item);
             // The softmax has read the previous item's O.  Waited for at every
             // item, an empty one included, so that ODONE never completes a
             // second phase before the softmax has seen the first (a parity
@@ -550,16 +578,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             *reinterpret_cast<uint4*>(smem + C::OFF_Q + off) = make_uint4(0, 0, 0, 0);
         __syncwarp();
         for (int k = 0;; ++k) {
-            const int item = take_item(k);
-            if (item < 0) break;
-            const ItemInfo it = item_info<D>(P, tp, item);
+            const ItemInfo it = take_item(k);
+            if (it.item < 0) break;
+            const int nrows = it.nblk > 0 ? it.nseq * P.G : 0;   // an empty split reads no Q
             const int qb = C::NQ == 2 ? (k & 1) : 0;
             const uint32_t quse = uint32_t(C::NQ == 2 ? k >> 1 : k);
             if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::QEMPTY + qb), (quse & 1u) ^ 1u, s_abort, P.err, kErrWaitQ)))
                 break;
             const uint32_t q_s = sbase + C::OFF_Q + qb * C::Q_BYTES;
-            // an empty split reads no Q
-            const int nrows = it.nblk > 0 ? it.nseq * P.G : 0;
 #pragma unroll 1
             for (int row = lane; row < nrows; row += 32) {
                 const int s = P.group_seqs[it.first + row / P.G];
@@ -580,7 +606,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ------------------------------------------------ softmax / epilogue
         const int wg = (warp - 4) / 4;                 // 0: first half of each block's keys, 1: second half
         const int quarter = warp & 3;                  // TMEM lane quarter this warp may access
-        const int row = quarter * 32 + lane;           // == TMEM lane of this thread's row
         const uint32_t lane_base = uint32_t(quarter * 32) << 16;
         float* xmax = reinterpret_cast<float*>(smem + C::OFF_X);          // [2][2][128]
         float* xl = xmax + 2 * 2 * kRows;                                 // [2][2][128]
@@ -588,23 +613,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float2 c2 = make_float2(c, c);
         const float neg = c >= 0.f ? -INFINITY : INFINITY;     // a raw logit that weighs nothing
         const bool zero_scale = c == 0.f;                      // then neg * c is not -inf
-        bool ok = true;
+        constexpr int KPT = C::KPT;                    // keys of this thread per block
+        constexpr int SEG = KPT / 2;                   // keys per row-sum segment
+        const int row = quarter * 32 + lane;           // == TMEM lane of this thread's row
         int jg = 0;
         for (int k = 0;; ++k) {
-            const int item = take_item(k);
-            if (item < 0) {
-                ok = item == -1;
-                break;
-            }
-            const ItemInfo it = item_info<D>(P, tp, item);
+            const ItemInfo it = take_item(k);
+            if (it.item < 0) break;
             const int nrows = it.nseq * P.G;
             const bool rows = quarter * 32 < nrows;    // warp-uniform
             const bool valid = row < nrows;
-            int orow = 0;
-            if (valid) {
-                const int s = P.group_seqs[it.first + row / P.G];
-                orow = s * P.Hq + it.h * P.G + row % P.G;
-            }
+            // the row's sequence: loaded now, needed only at the item's end
+            const int seq = valid ? P.group_seqs[it.first + row / P.G] : 0;
             // delta mode: the bits of the positions this row's donor
             // encodes (they come from the delta rows, not from this span)
             const uint32_t* mrow = nullptr;
@@ -614,7 +634,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mrow = P.dmask + size_t(((long(it.prompt) * P.Dst + (mid - 1)) * P.N + P.layer) * P.Hkv + it.h) *
                                          size_t(P.delta_w32);
             }
-            float m_run = -INFINITY, l_run = 0.f;
+            // row sum kept per segment of this thread's keys (two), added at
+            // the item's end
+            float m_run = -INFINITY, l_seg0 = 0.f, l_seg1 = 0.f;
+            bool ok = true;
             for (int j = 0; j < it.nblk; ++j, ++jg) {
                 const int slot = jg % NSLOT;
                 // waits are made warp-uniform: tcgen05.ld/st are warp-collective
@@ -623,18 +646,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ok = false;
                     break;
                 }
-                const uint32_t s_col = tmem + lane_base + col_s(jg) + wg * C::KPT;
-                const int kbase = it.k0 + j * C::BN + wg * C::KPT;
-                float s[C::KPT];
+                const uint32_t s_col = tmem + lane_base + col_s(jg) + wg * KPT;
+                const int kbase = it.k0 + j * C::BN + wg * KPT;
+                float s[KPT];
                 float e0 = 0.f;
                 // keys of this half that do not count: past the split's end,
                 // and the positions this row's donor encodes
-                uint32_t dead[C::KPT / 32];
+                uint32_t dead[KPT / 32];
                 bool any_dead = false;
                 if (rows) {
                     tc::tc_fence_after();
 #pragma unroll
-                    for (int q = 0; q < C::KPT / 32; ++q) {
+                    for (int q = 0; q < KPT / 32; ++q) {
                         float v[32];
                         tc::tmem_ld32(s_col + q * 32, v);
 #pragma unroll
@@ -642,7 +665,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     uint32_t anyd = 0u;
 #pragma unroll
-                    for (int q = 0; q < C::KPT / 32; ++q) {
+                    for (int q = 0; q < KPT / 32; ++q) {
                         const int live = it.k1 - (kbase + 32 * q);
                         dead[q] = live >= 32 ? 0u : (live <= 0 ? 0xffffffffu : (0xffffffffu << live));
                         if (mrow) dead[q] |= __ldg(mrow + (kbase >> 5) + q);
@@ -652,7 +675,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tc::tmem_wait_ld();
                     if (any_dead) {
 #pragma unroll
-                        for (int i = 0; i < C::KPT; ++i)
+                        for (int i = 0; i < KPT; ++i)
                             if ((dead[i >> 5] >> (i & 31)) & 1u) s[i] = neg;
                     }
                     // extreme of this half's raw logits (max for c >= 0)
@@ -660,7 +683,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     e0 = s[0];
                     if (c >= 0.f) {
 #pragma unroll
-                        for (int i = 4; i < C::KPT; i += 4) {
+                        for (int i = 4; i < KPT; i += 4) {
                             e0 = fmaxf(e0, s[i]);
                             e1 = fmaxf(e1, s[i + 1]);
                             e2 = fmaxf(e2, s[i + 2]);
@@ -669,7 +692,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         e0 = fmaxf(fmaxf(e0, e1), fmaxf(e2, e3));
                     } else {
 #pragma unroll
-                        for (int i = 4; i < C::KPT; i += 4) {
+                        for (int i = 4; i < KPT; i += 4) {
                             e0 = fminf(e0, s[i]);
                             e1 = fminf(e1, s[i + 1]);
                             e2 = fminf(e2, s[i + 2]);
@@ -684,7 +707,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 xm[wg * kRows + row] = e0;
                 const uint32_t xch = bar(Bb::XCH + 4 * (jg & 1) + quarter);
                 tc::mbar_arrive(xch);
-                if (!__all_sync(0xffffffffu, tc::mbar_wait(xch, uint32_t(jg >> 1) & 1u, s_abort, P.err, kErrWaitSoftmax))) {
+                if (!__all_sync(0xffffffffu,
+                                tc::mbar_wait(xch, uint32_t(jg >> 1) & 1u, s_abort, P.err, kErrWaitSoftmax))) {
                     ok = false;
                     break;
                 }
@@ -702,31 +726,35 @@ __global__ void __launch_bounds__(kThreads, 1)
                     // finite reference makes the dead keys' weights 0
                     const float mref = m_run == -INFINITY ? 0.f : m_run;
                     const float2 nm2 = make_float2(-mref, -mref);
-                    float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
-                    uint32_t pk[C::KPT / 2];
+                    // per segment: exponentials, the segment's row sum, and
+                    // its P (bf16 pairs) stored over the first columns of
+                    // this half of the slot
 #pragma unroll
-                    for (int i = 0; i < C::KPT / 2; ++i) {
-                        const float2 z = __ffma2_rn(make_float2(s[2 * i], s[2 * i + 1]), c2, nm2);
-                        float2 e = make_float2(ex2(z.x), ex2(z.y));
-                        if (any_dead && zero_scale) {
-                            e.x = ((dead[(2 * i) >> 5] >> ((2 * i) & 31)) & 1u) ? 0.f : e.x;
-                            e.y = ((dead[(2 * i + 1) >> 5] >> ((2 * i + 1) & 31)) & 1u) ? 0.f : e.y;
+                    for (int g = 0; g < 2; ++g) {
+                        float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
+                        uint32_t pk[SEG / 2];
+#pragma unroll
+                        for (int i = 0; i < SEG / 2; ++i) {
+                            const int pi = g * (SEG / 2) + i;
+                            const float2 z = __ffma2_rn(make_float2(s[2 * pi], s[2 * pi + 1]), c2, nm2);
+                            float2 e = make_float2(ex2(z.x), ex2(z.y));
+                            if (any_dead && zero_scale) {
+                                e.x = ((dead[(2 * pi) >> 5] >> ((2 * pi) & 31)) & 1u) ? 0.f : e.x;
+                                e.y = ((dead[(2 * pi + 1) >> 5] >> ((2 * pi + 1) & 31)) & 1u) ? 0.f : e.y;
+                            }
+                            if (i & 1)
+                                acc1 = __fadd2_rn(acc1, e);
+                            else
+                                acc0 = __fadd2_rn(acc0, e);
+                            const __nv_bfloat162 h2 = __floats2bfloat162_rn(e.x, e.y);
+                            pk[i] = *reinterpret_cast<const uint32_t*>(&h2);
                         }
-                        if (i & 1)
-                            acc1 = __fadd2_rn(acc1, e);
+                        const float ls = (acc0.x + acc1.x) + (acc0.y + acc1.y);
+                        if (g == 0)
+                            l_seg0 = l_seg0 * alpha + ls;
                         else
-                            acc0 = __fadd2_rn(acc0, e);
-                        const __nv_bfloat162 h2 = __floats2bfloat162_rn(e.x, e.y);
-                        pk[i] = *reinterpret_cast<const uint32_t*>(&h2);
-                    }
-                    l_run = l_run * alpha + ((acc0.x + acc1.x) + (acc0.y + acc1.y));
-                    // P (bf16 pairs) over the first columns of this half of the slot
-#pragma unroll
-                    for (int q = 0; q < C::KPT / 32; ++q) {
-                        uint32_t part[16];
-#pragma unroll
-                        for (int i = 0; i < 16; ++i) part[i] = pk[q * 16 + i];
-                        tmem_st16(s_col + q * 16, part);
+                            l_seg1 = l_seg1 * alpha + ls;
+                        store_p(s_col + g * (SEG / 2), pk);
                     }
                     if (__any_sync(0xffffffffu, resc)) {
                         // O must hold P V of every earlier block of this item
@@ -762,13 +790,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             // ---- epilogue: partial state of this row for this item ----
             // Every thread waits for the item's O before it frees it, so
             // arrivals of one item never land in an earlier item's phase.
-            if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::ODONE), uint32_t(k) & 1u, s_abort, P.err,
-                                                       kErrWaitSoftmax))) {
-                ok = false;
+            if (!__all_sync(0xffffffffu,
+                            tc::mbar_wait(bar(Bb::ODONE), uint32_t(k) & 1u, s_abort, P.err, kErrWaitSoftmax)))
                 break;
-            }
             tc::tc_fence_after();
+            const int orow = seq * P.Hq + it.h * P.G + row % P.G;
             const size_t idx = size_t(it.split) * P.B * P.Hq + size_t(orow);
+            float* xb = xl + (k & 1) * (2 * kRows);
             if (it.nblk > 0) {
                 if (rows) {
                     float* op = P.ws_o + idx * D + wg * C::OCH;
@@ -785,25 +813,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                     }
                 }
-                // a row's sum is the sum of its two halves' sums
-                float* xb = xl + (k & 1) * (2 * kRows);
-                xb[wg * kRows + row] = l_run;
+                // a row's sum: its segments' sums in key order, then the two
+                // halves
+                xb[wg * kRows + row] = l_seg0 + l_seg1;
                 tc::mbar_arrive(bar(Bb::LXCH));
-                if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::LXCH), uint32_t(k) & 1u, s_abort, P.err,
-                                                           kErrWaitSoftmax))) {
-                    ok = false;
+                if (!__all_sync(0xffffffffu,
+                                tc::mbar_wait(bar(Bb::LXCH), uint32_t(k) & 1u, s_abort, P.err, kErrWaitSoftmax)))
                     break;
-                }
                 if (wg == 0 && valid) P.ws_ml[idx] = make_float2(m_run, xb[row] + xb[kRows + row]);
             } else {
                 // an empty split: a state with no keys (still one exchange
                 // round, so every item moves the exchange barrier once)
                 tc::mbar_arrive(bar(Bb::LXCH));
-                if (!__all_sync(0xffffffffu, tc::mbar_wait(bar(Bb::LXCH), uint32_t(k) & 1u, s_abort, P.err,
-                                                           kErrWaitSoftmax))) {
-                    ok = false;
+                if (!__all_sync(0xffffffffu,
+                                tc::mbar_wait(bar(Bb::LXCH), uint32_t(k) & 1u, s_abort, P.err, kErrWaitSoftmax)))
                     break;
-                }
                 if (wg == 0 && valid) P.ws_ml[idx] = make_float2(-INFINITY, 0.f);
             }
             tc::tc_fence_before();
@@ -814,16 +838,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc::tc_fence_after();
     if (warp == 1) tc::tmem_dealloc(tmem, kTmemCols);
-    // This CTA's work is done: the merge queued behind this grid may launch
-    // (it waits for the whole grid before it reads anything).  Every CTA of
-    // this grid is running by the time all of them have signalled, so the
-    // merge's CTAs never hold an SM this grid still needs.
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-    // Launched right behind the generated-span pass, this grid may start
-    // while that pass's last CTAs still run (it reads nothing they write);
-    // waiting for it here makes this grid's completion imply that pass's, so
-    // the merge that follows sees both.  A no-op for a plain launch.
-    asm volatile("griddepcontrol.wait;" ::: "memory");
+    if (P.prefix_after_gs) {
+        // This CTA's work is done: the merge queued behind this grid may
+        // launch (it waits for the whole grid before it reads anything).
+        // Every CTA of this grid is running by the time all of them have
+        // signalled, so the merge's CTAs never hold an SM it still needs.
+        asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+        // Launched right behind the generated-span pass, this grid may start
+        // while that pass's last CTAs still run (it reads nothing they
+        // write); waiting for it here makes this grid's completion imply that
+        // pass's, so the merge that follows sees both.
+        asm volatile("griddepcontrol.wait;" ::: "memory");
+    }
     // The last CTA to finish resets the work counter for the next launch
     // (every CTA has claimed its last item before it gets here).
     if (threadIdx.x == 0) {
@@ -907,14 +933,13 @@ int prefix_tc_splits(int d, int p_vis, int max_splits, int* bounds) {
     // Splits depend only on the visible span length (and the cap), so a
     // row's arithmetic never depends on which other rows share its tile or
     // launch.  Every item gathers its tile's queries and stores its partial
-    // states, so fewer, longer items move fewer bytes: splits of kSplitKeys
+    // states, so fewer, longer items move fewer bytes: splits of kPrefixSplitKeys
     // keys, all but the last full.  A longer span ends in a shorter split,
     // which the split-major item order hands out last, so a launch ends on
     // short items.  Past the cap, the blocks are shared out evenly.
-    constexpr int kSplitKeys = 3072;
     const int bn = prefix_tc_box_rows(d);
     const int nb = (p_vis + bn - 1) / bn;
-    const int full = kSplitKeys / bn;
+    const int full = kPrefixSplitKeys / bn;
     int ns = (nb + full - 1) / full;
     bounds[0] = 0;
     if (ns <= max_splits) {

@@ -3,9 +3,11 @@
 // decode step attends over the prompt span and the t generated entries).
 //
 // HBM-bound streaming kernel:
-//   * persistent warps, each walking a fixed stream of work items
-//     (sequence, kv head, row chunk, key split) and, inside an item, blocks
-//     of 16 keys;
+//   * persistent warps walking work items (sequence, kv head, row chunk, key
+//     split) and, inside an item, blocks of 16 keys: a fixed stream per warp
+//     when this pass goes first, items claimed at run time (one ahead) when
+//     it runs behind the prompt-span pass, so warps that start late (on SMs
+//     that pass still holds) simply take fewer;
 //   * every block's K and V rows (contiguous in the generated-span store) are
 //     fetched by one bulk async copy (cp.async.bulk, mbarrier-tracked) into a
 //     two-stage per-warp ring; the next block -- of this item or the next one
@@ -84,7 +86,8 @@ struct GS {
     static constexpr uint32_t OFF_RED = 2 * STAGE;
     static constexpr uint32_t OFF_PP = OFF_RED + KPW * GSTRIDE * 4;
     static constexpr uint32_t OFF_BAR = OFF_PP + KPW * NV * 8;
-    static constexpr uint32_t PER_WARP = (OFF_BAR + 16 + 127) / 128 * 128;
+    static constexpr uint32_t OFF_TAKEN = OFF_BAR + 16;       // [4] items in the order the issue cursor took them
+    static constexpr uint32_t PER_WARP = (OFF_TAKEN + 16 + 127) / 128 * 128;
     static constexpr uint32_t SMEM = WARPS * PER_WARP;
     static_assert(NV % 4 == 0 || NV < 4, "reduce layout");
     static_assert(NV < LPK || NV == VPL * LPK, "every logit of a group owned by one lane");
@@ -98,13 +101,13 @@ struct Item {
     int s, h, rc, split, k0, k1, nblk;
 };
 
+// Work item idx = ((sequence * Hkv + kv head) * row chunks + row chunk) *
+// splits + key split.
 template <int D, int GT>
-__device__ __forceinline__ bool item_at(const AttnParams& P, int idx, int n_items, Item& it) {
-    if (idx >= n_items) return false;
+__device__ __forceinline__ void item_of(const AttnParams& P, int idx, Item& it) {
     const int n_rc = P.G / GT;
-    int rem = idx;
-    it.split = rem % P.nss;
-    rem /= P.nss;
+    it.split = idx % P.nss;
+    int rem = idx / P.nss;
     it.rc = rem % n_rc;
     rem /= n_rc;
     it.h = rem % P.Hkv;
@@ -115,7 +118,6 @@ __device__ __forceinline__ bool item_at(const AttnParams& P, int idx, int n_item
     it.k0 = P.s_lo + it.split * P.s_chunk;
     it.k1 = min(P.s_hi, it.k0 + P.s_chunk);
     it.nblk = it.k1 > it.k0 ? (it.k1 - it.k0 + 15) / 16 : 0;
-    return true;
 }
 
 template <int D, int GT>
@@ -124,27 +126,30 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
     using C = GS<D, GT>;
     extern __shared__ __align__(128) uint8_t smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // Launched as a programmatic dependent of whatever precedes it on the
-    // stream, this grid may start before that grid has finished: wait for it
-    // (its writes visible) before reading or writing anything.  A no-op for a
-    // plain launch.  Only then may the prompt-span pass queued behind this
-    // grid start: it reads the queries and the prompt stores without a wait
-    // of its own, so its start must imply that everything before this grid
-    // on the stream is complete.  It reads nothing this grid writes, so it
-    // may take the SMs this grid's last CTAs leave idle.
-    asm volatile("griddepcontrol.wait;" ::: "memory");
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    // The call's first pass: launched as a programmatic dependent of
+    // whatever precedes it on the stream, this grid may start before that
+    // work has finished, so it waits for it (its writes visible) before
+    // reading or writing anything.  Only then may the pass queued behind it
+    // launch: the prompt-span pass reads the queries and the prompt stores
+    // without a wait of its own, and it reads nothing this grid writes, so it
+    // may take the SMs this grid's last CTAs leave.  (Behind the prompt-span
+    // pass instead, that pass has waited before it let this grid launch, and
+    // this grid reads nothing it writes; see the end of the kernel.)  No-ops
+    // for a plain launch.
+    if (!P.gs_after_prefix) {
+        asm volatile("griddepcontrol.wait;" ::: "memory");
+        asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    }
     uint8_t* ws = smem + warp * C::PER_WARP;
     const uint32_t wbase = tc::smem_u32(ws);
     const uint32_t bar0 = wbase + C::OFF_BAR;
     float* red = reinterpret_cast<float*>(ws + C::OFF_RED);
     float2* pp = reinterpret_cast<float2*>(ws + C::OFF_PP);
+    int* taken_items = reinterpret_cast<int*>(ws + C::OFF_TAKEN);
 
     const int gi = lane / C::LPK, dl = lane % C::LPK;
     const int g_mine = dl % GT;
     const int c0 = dl, c1 = dl + C::LPK;
-    const int gwarp = blockIdx.x * C::WARPS + warp;
-    const int nwarps = gridDim.x * C::WARPS;
     volatile int abort_flag = 0;
 
     if (lane == 0) {
@@ -154,14 +159,53 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
     }
     __syncwarp();
 
-    // ---- issue cursor: walks (item, block) units of this warp's stream ----
+    // ---- work items: warp w of the grid starts on item w.  As the call's
+    // first pass (all warps start together) it then walks items w + k *
+    // (warps of the grid): the extra items of an uneven share land on the
+    // first CTAs, so the other SMs come free whole and early for the
+    // prompt-span pass queued behind.  Behind the prompt-span pass (CTAs
+    // start as that pass's CTAs leave) every later item is claimed from the
+    // launch-wide counter (numbered from the grid's warp count on), one
+    // ahead: lane 0 holds the claim in flight, whose value is needed only
+    // when the next item starts ----
+    const unsigned nwarps = gridDim.x * C::WARPS;
+    const int first_item = int(blockIdx.x * C::WARPS + warp);
+    const bool claims = P.gs_after_prefix != 0;
+    unsigned claim = unsigned(first_item) + nwarps;
+    if (claims && lane == 0) claim = nwarps + atomicAdd(P.sched + 2, 1u);
+    auto next_item = [&]() -> int {
+        const int i = int(__shfl_sync(kFull, claim, 0));
+        if (i >= n_items) return -1;
+        if (claims) {
+            if (lane == 0) claim = nwarps + atomicAdd(P.sched + 2, 1u);
+        } else {
+            claim += nwarps;
+        }
+        return i;
+    };
+
+    // ---- issue cursor: walks (item, block) in claim order and records every
+    // item it takes (then -1) for the consumer.  It runs two blocks ahead and
+    // every item has a block (the host keeps at least 64 keys per split), so
+    // it is at most two items ahead ----
     Item iss;
-    int iss_idx = gwarp, iss_b = 0;
-    bool iss_ok = item_at<D, GT>(P, iss_idx, n_items, iss);
-    while (iss_ok && iss.nblk == 0) {
-        iss_idx += nwarps;
-        iss_ok = item_at<D, GT>(P, iss_idx, n_items, iss);
-    }
+    int iss_idx = first_item < n_items ? first_item : -1, iss_b = 0, recorded = 1;
+    if (lane == 0) taken_items[0] = iss_idx;
+    bool iss_ok = false;
+    auto seek = [&]() {   // the first block at or after item iss_idx
+        iss_ok = false;
+        while (iss_idx >= 0) {
+            item_of<D, GT>(P, iss_idx, iss);
+            if (iss.nblk > 0) {
+                iss_ok = true;
+                return;
+            }
+            iss_idx = next_item();
+            if (lane == 0) taken_items[recorded & 3] = iss_idx;
+            ++recorded;
+        }
+    };
+    seek();
     int issued = 0;
     const uint64_t pol = l2_evict_first_policy();
     auto issue_next = [&]() {
@@ -184,10 +228,10 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
         ++issued;
         if (++iss_b >= iss.nblk) {
             iss_b = 0;
-            do {
-                iss_idx += nwarps;
-                iss_ok = item_at<D, GT>(P, iss_idx, n_items, iss);
-            } while (iss_ok && iss.nblk == 0);
+            iss_idx = next_item();
+            if (lane == 0) taken_items[recorded & 3] = iss_idx;
+            ++recorded;
+            seek();
         }
     };
     issue_next();
@@ -195,8 +239,12 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
 
     int consumed = 0;
     bool ok = true;
-    Item it;
-    for (int idx = gwarp; ok && item_at<D, GT>(P, idx, n_items, it); idx += nwarps) {
+    for (int taken = 0; ok; ++taken) {
+        __syncwarp();
+        const int idx = taken_items[taken & 3];
+        if (idx < 0) break;
+        Item it;
+        item_of<D, GT>(P, idx, it);
         // q rows of this item, pre-scaled into log2 units, as dim pairs
         float2 q2[GT][8];
 #pragma unroll
@@ -440,6 +488,27 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
         volatile int no_abort = 0;
         tc::mbar_wait(bar0 + 8 * (consumed & 1), uint32_t(consumed >> 1) & 1u, &no_abort, P.err, kErrWaitGsDrain,
                       10000000000ull);
+    }
+    if (P.gs_after_prefix) {
+        // Behind the prompt-span pass: this grid's completion must imply that
+        // pass's, so the merge queued behind this grid sees both.  Then the
+        // merge may launch (it waits for this whole grid before it reads
+        // anything); every CTA of this grid is running by the time all of
+        // them have signalled, so the merge's CTAs never hold an SM it still
+        // needs.
+        asm volatile("griddepcontrol.wait;" ::: "memory");
+        asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    }
+    // Run-time claims: the last warp to finish resets the item counter for
+    // the next launch (every warp's claims have all returned before it gets
+    // here: the one in flight when its last item started came back past the
+    // end and ended its walk).
+    if (claims && lane == 0) {
+        __threadfence();
+        if (atomicAdd(P.sched + 3, 1u) == nwarps - 1) {
+            atomicExch(P.sched + 2, 0u);
+            atomicExch(P.sched + 3, 0u);
+        }
     }
 }
 

@@ -57,8 +57,9 @@ std::string build_plan(const splice_model_shape& sh, int P, int Tp, int Dslots, 
 
     // stored-donor index of every slot (the non-ZERO slots in slot order)
     std::vector<int> stored(Dslots, -1);
-    for (int k = 0, n = 0; k < Dslots; ++k)
-        if (kinds[k] != SPLICE_DONOR_ZERO) stored[k] = n++;
+    int n_stored = 0;
+    for (int k = 0; k < Dslots; ++k)
+        if (kinds[k] != SPLICE_DONOR_ZERO) stored[k] = n_stored++;
 
     plan.src.assign(size_t(plan.num_tables) * B, 0);
     plan.table_group_off.assign(plan.num_tables + 1, 0);
@@ -120,11 +121,22 @@ std::string build_plan(const splice_model_shape& sh, int P, int Tp, int Dslots, 
                     plan.group_seqs.push_back(std::get<4>(keyed[k]));
                     plan.group_mask.push_back(std::get<3>(keyed[k]));
                 }
+                // the tile's store and its span base index: kind 0 = clean
+                // span (base = prompt), 1 = stored donor span, 2 = a donor's
+                // delta rows (base = prompt * stored slots + stored index);
+                // the span of (layer l, kv head h) is (base * N + l) * Hkv + h
+                const int gsrc = std::get<2>(keyed[i]);
+                const int gprompt = std::get<1>(keyed[i]);
+                int kind = 0, base = gprompt;
+                if (gsrc != int(SPLICE_SRC_CLEAN)) {
+                    kind = (gsrc & kGroupDelta) ? 2 : 1;
+                    base = gprompt * n_stored + stored[(gsrc & 0xff) - int(SPLICE_SRC_DONOR0)];
+                }
                 for (int off = 0; off < int(j - i); off += plan.seqs_per_tile) {
                     plan.tiles.push_back(gid);
                     plan.tiles.push_back(first + off);
                     plan.tiles.push_back(std::min(plan.seqs_per_tile, int(j - i) - off));
-                    plan.tiles.push_back(0);
+                    plan.tiles.push_back((base << 2) | kind);
                     if (std::get<0>(keyed[i]) == 0) ++span_tiles;
                 }
                 i = j;

@@ -20,6 +20,8 @@ constexpr int kMaxSuffixSplits = 8;
 constexpr int kMaxSplits = kMaxPrefixSplits + kMaxSuffixSplits;
 // Rows of one tensor-core prefix tile (tcgen05 M).
 constexpr int kTileRows = 128;
+// Keys of a full prompt-span split (every split of a span but its last).
+constexpr int kPrefixSplitKeys = 3072;
 // Group source flag: the group reads the delta-encoded rows of a donor slot
 // (group_src = kGroupDelta | (SPLICE_SRC_DONOR0 + slot)).
 constexpr int32_t kGroupDelta = SPLICE_GROUP_DELTA;
@@ -52,7 +54,7 @@ struct Plan {
     std::vector<int32_t> group_mask;        // parallel to group_seqs: 0, or stored slot + 1 (delta rows)
     // Row tiles of at most kTileRows rows (seqs_per_tile sequences x G heads).
     std::vector<int32_t> table_tile_off;    // [num_tables + 1]
-    std::vector<int32_t> tiles;             // [tiles][4]: group, first, count, 0
+    std::vector<int32_t> tiles;             // [tiles][4]: group, first, count, (span base << 2) | store kind
     std::vector<int32_t> table_span_tiles;  // [num_tables] tiles of stored-span groups (the rest read delta rows)
     int seqs_per_tile = 0;
 
@@ -105,7 +107,8 @@ struct AttnParams {
     const int32_t* dcount;        // [P][Dst][N][Hkv] encoded rows per span
     const int32_t* slot_delta;    // [num_slots] 1 = the slot is read in delta mode
     unsigned* err;
-    unsigned* sched;              // [2] prompt-span work counter and finished-CTA count, zero between launches
+    unsigned* sched;              // [4] prompt-span work counter and finished-CTA count, generated-span unit
+                                  // counter and finished-CTA count; zero between launches
     int B, N, Hq, Hkv, D, G, Tp, T, Dst;
     int layer, step;
     int p_lo, p_hi, s_lo, s_hi;
@@ -113,6 +116,8 @@ struct AttnParams {
     int nsd;                      // splits of the delta rows (delta mode)
     int delta_on, delta_w32;
     int fuse_append;              // the generated-span pass also appends entry step - 1 (see kn, vn)
+    int gs_after_prefix;          // the generated-span pass runs behind the prompt-span pass of the call
+    int prefix_after_gs;          // the prompt-span pass runs behind the generated-span pass of the call
     int p_chunk, s_chunk;         // keys per split
     int n_tiles;
     int n_span_tiles;             // tiles [0, n_span_tiles) read stored spans, the rest delta rows
@@ -130,12 +135,17 @@ int desc_device(const splice_desc* d);
 int launch_append(const uint16_t* kn, const uint16_t* vn, uint16_t* ks, uint16_t* vs, int B,
                   int N, int Hkv, int D, int T, int layer, int step, void* stream);
 // overlap_previous: launched as a programmatic dependent of the preceding
-// work on the stream (the kernel waits for it before reading or writing
-// anything, and lets its own dependents launch only after that wait).
+// work on the stream.  With p.gs_after_prefix = 0 the kernel is the call's
+// first and waits for that work before reading or writing anything, then
+// lets its dependents launch.  With 1 it directly follows the prompt-span
+// pass of the same call, which has already waited; it reads nothing that
+// pass writes, waits for it only before it exits, and lets its own
+// dependents launch only once its work is done.
 int launch_generated_span(const AttnParams& p, void* stream, bool overlap_previous);
 int generated_span_resident_warps(int d);
-// overlap_previous: the launch directly follows the prompt-span pass on the
-// same stream (programmatic dependent launch; the kernel waits for it).
+// overlap_previous: the launch directly follows the last pass of the same
+// call on the stream (programmatic dependent launch; the kernel waits for it,
+// and that pass's completion implies the other pass's).
 int launch_merge(const AttnParams& p, void* stream, bool overlap_previous);
 
 // A copy of `bytes` (a multiple of 16) from src to dst by a kernel that lets
@@ -155,10 +165,14 @@ int prefix_tc_box_rows(int d);
 int prefix_tc_splits(int d, int p_vis, int max_splits, int* bounds);
 // maps: six tensor maps -- clean K, V; donor K, V; delta rows K, V.
 // bounds: the span splits (p.nsp + 1 values); delta_keys: keys per split of
-// the delta rows.  overlap_previous: the launch directly follows the
-// generated-span pass on the same stream and may start while that pass
-// finishes (programmatic dependent launch); the kernel waits for it before
-// it exits.
+// the delta rows.  overlap_previous: a programmatic dependent launch of the
+// preceding work on the stream.  With p.prefix_after_gs = 0 the kernel is
+// the call's first: it waits for that work before it reads anything, then
+// lets its dependents (the generated-span pass) launch onto the SMs its CTAs
+// leave.  With 1 it directly follows the generated-span pass of the call,
+// which has already waited and lets it start on the SMs that pass's last
+// CTAs leave; it reads nothing that pass writes and waits for it before it
+// exits.
 int launch_prefix_tc(const AttnParams& p, const void* maps, const int* bounds, int delta_keys, void* stream,
                      bool overlap_previous);
 
