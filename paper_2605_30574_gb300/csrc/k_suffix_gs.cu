@@ -11,7 +11,9 @@
 //   * every block's K and V rows (contiguous in the generated-span store) are
 //     fetched by one bulk async copy (cp.async.bulk, mbarrier-tracked) into a
 //     two-stage per-warp ring; the next block -- of this item or the next one
-//     -- is in flight while the current one is computed;
+//     -- is in flight while the current one is computed; an item's first
+//     block brings the item's query rows with it, so no item starts on a
+//     load from global memory;
 //   * a key row of d values is split over LPK = d / 16 lanes (16 dims each,
 //     two 16-byte chunks); q . k partial sums are reduced across the LPK
 //     lanes through a small shared-memory transpose (lane dl of a key group
@@ -66,6 +68,14 @@ __device__ __forceinline__ void bulk_copy(uint32_t dst, const void* src, uint32_
         : "memory");
 }
 
+// The same without a cache hint: the query rows are read again by the
+// prompt-span pass of the call.
+__device__ __forceinline__ void bulk_copy_plain(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                 "l"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+
 template <int D, int GT>
 struct GS {
     static constexpr int LPK = D / 16;              // lanes per key
@@ -87,7 +97,9 @@ struct GS {
     static constexpr uint32_t OFF_PP = OFF_RED + KPW * GSTRIDE * 4;
     static constexpr uint32_t OFF_BAR = OFF_PP + KPW * NV * 8;
     static constexpr uint32_t OFF_TAKEN = OFF_BAR + 16;       // [4] items in the order the issue cursor took them
-    static constexpr uint32_t PER_WARP = (OFF_TAKEN + 16 + 127) / 128 * 128;
+    static constexpr uint32_t QROWS = GT * D * 2;             // the GT query rows of one item
+    static constexpr uint32_t OFF_Q = OFF_TAKEN + 16;         // [2] query rows, brought with each item's first block
+    static constexpr uint32_t PER_WARP = (OFF_Q + 2 * QROWS + 127) / 128 * 128;
     static constexpr uint32_t SMEM = WARPS * PER_WARP;
     static_assert(NV % 4 == 0 || NV < 4, "reduce layout");
     static_assert(NV < LPK || NV == VPL * LPK, "every logit of a group owned by one lane");
@@ -206,11 +218,14 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
         }
     };
     seek();
-    int issued = 0;
+    int issued = 0, iss_items = 0;
     const uint64_t pol = l2_evict_first_policy();
     auto issue_next = [&]() {
         if (!iss_ok) return;
         const int stg = issued & 1;
+        // an item's first block also brings the item's GT query rows
+        // (contiguous in q) into the item's query buffer
+        const bool first = iss_b == 0;
         const int j = iss.k0 + iss_b * 16;
         int nk = min(16, iss.k1 - j);
         // fused append: entry step - 1 (the block's last row) is not in the
@@ -219,13 +234,17 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
         const uint32_t bytes = uint32_t(nk) * C::ROW;
         if (lane == 0) {
             const uint32_t dst = wbase + stg * C::STAGE;
-            tc::mbar_arrive_expect_tx(bar0 + 8 * stg, 2 * bytes);
+            tc::mbar_arrive_expect_tx(bar0 + 8 * stg, 2 * bytes + (first ? C::QROWS : 0u));
+            if (first)
+                bulk_copy_plain(wbase + C::OFF_Q + (iss_items & 1) * C::QROWS,
+                                P.q + (size_t(iss.s) * P.Hq + iss.h * P.G + iss.rc * GT) * D, C::QROWS, bar0 + 8 * stg);
             if (bytes) {
                 bulk_copy(dst, iss.k + size_t(j) * D, bytes, bar0 + 8 * stg, pol);
                 bulk_copy(dst + C::BK * C::ROW, iss.v + size_t(j) * D, bytes, bar0 + 8 * stg, pol);
             }
         }
         ++issued;
+        if (first) ++iss_items;
         if (++iss_b >= iss.nblk) {
             iss_b = 0;
             iss_idx = next_item();
@@ -237,7 +256,7 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
     issue_next();
     issue_next();
 
-    int consumed = 0;
+    int consumed = 0, cons_items = 0;
     bool ok = true;
     for (int taken = 0; ok; ++taken) {
         __syncwarp();
@@ -245,12 +264,22 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
         if (idx < 0) break;
         Item it;
         item_of<D, GT>(P, idx, it);
-        // q rows of this item, pre-scaled into log2 units, as dim pairs
+        // q rows of this item, pre-scaled into log2 units, as dim pairs: in
+        // the item's query buffer once its first block has landed
         float2 q2[GT][8];
+        if (it.nblk > 0) {
+            const bool got = tc::mbar_wait(bar0 + 8 * (consumed & 1), uint32_t(consumed >> 1) & 1u, &abort_flag,
+                                           P.err, kErrWaitGs);
+            if (!__all_sync(kFull, got)) {
+                ok = false;
+                break;
+            }
+        }
+        const uint8_t* qsm = ws + C::OFF_Q + (cons_items & 1) * C::QROWS;
+        if (it.nblk > 0) ++cons_items;
 #pragma unroll
         for (int g = 0; g < GT; ++g) {
-            const int hq = it.h * P.G + it.rc * GT + g;
-            const uint4* qr = reinterpret_cast<const uint4*>(P.q + (size_t(it.s) * P.Hq + hq) * D);
+            const uint4* qr = reinterpret_cast<const uint4*>(qsm + g * D * 2);
             const uint4 a = qr[c0], b = qr[c1];
             const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
 #pragma unroll
