@@ -59,7 +59,8 @@ NOMINAL_HBM_GBS = 8000.0
 # reduced ladder case (read + written bytes / algorithmic bytes of that launch);
 # traffic grows in proportion to the units a launch processes.  Only kernels
 # whose current build was captured are listed.
-TRAFFIC_PER_ALGORITHMIC_BYTE = {"generated_span_pass": 545.24 / 538.97}
+TRAFFIC_PER_ALGORITHMIC_BYTE = {"generated_span_pass": (539.054 + 6.104) / 541.065,
+                                "prompt_span_pass": (236.987 + 2.962) / 234.881}
 
 
 def step_schedule(T: int, n: int, offset: int = 0):
@@ -762,6 +763,12 @@ def profile_case(args):
                     base.scaffold_head, base.scaffold_tail, batch=args.batch_size,
                     sliding_window=base.sliding_window, global_every=base.global_every, sm_scale=base.sm_scale)
     sb = SweepBatch(wl, 0)
+    # algorithmic bytes of every launch of one repetition, for comparing a
+    # capture's DRAM counters with what the launch must move
+    for l in range(wl.num_layers):
+        ab = algorithmic_bytes(sb, l, args.step, fused=not args.unfused)
+        print(f"layer {l}: algorithmic bytes per launch " +
+              ", ".join(f"{k} {v}" for k, v in ab.items() if v))
     for _ in range(args.reps):
         for l in range(wl.num_layers):
             sb.gen_inputs(l, args.step)
