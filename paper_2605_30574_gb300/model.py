@@ -8,11 +8,11 @@ whole sweep batch at once.
   forward pass; its RoPE'd K and V fill the clean and donor stores the
   library reads, and the clean prompt's last logits give y_0.
 * Decode: each step t = 1 .. T-1 runs one forward pass of every sequence's
-  previous token y_{t-1} at position T_p + t - 1; at every layer the token's
-  K/V is appended to the generated-span store (``suffix_kv_append``) and the
-  query attends over its prompt span -- clean, donor or ZERO by the splice
-  rule l >= L and t >= W -- and its t generated entries
-  (``spliced_decode_attn``); the last layer's output gives y_t = argmax.
+  previous token y_{t-1} at position T_p + t - 1; at every layer one
+  ``spliced_decode_step`` call appends the token's K/V to the generated-span
+  store and lets the query attend over its prompt span -- clean, donor or
+  ZERO by the splice rule l >= L and t >= W -- and its t generated entries;
+  the last layer's output gives y_t = argmax.
   The replacement at t = W is not a copy: every sequence reads its source by
   reference, which is the same computation because the rule is monotone in t.
 
@@ -232,9 +232,9 @@ class SpliceDecode:
         h = model.embed[tokens].float()
         for l in range(dims.num_layers):
             q, k, v = model.qkv(l, h, pos)
-            S.suffix_kv_append(self.desc, l, t, k.contiguous(), v.contiguous(), self.k_suffix, self.v_suffix)
-            S.spliced_decode_attn(self.desc, l, t, q.contiguous(), self.k_clean, self.v_clean, self.k_donor,
-                                  self.v_donor, self.k_suffix, self.v_suffix, self.out, self.ws)
+            S.spliced_decode_step(self.desc, l, t, q.contiguous(), k.contiguous(), v.contiguous(), self.k_clean,
+                                  self.v_clean, self.k_donor, self.v_donor, self.k_suffix, self.v_suffix, self.out,
+                                  self.ws)
             h = model.block_out(l, h, self.out)
         return model.logits(h)
 
