@@ -57,6 +57,26 @@ __global__ void __launch_bounds__(256, 5) merge_kernel(AttnParams P) {
     }
 }
 
+// Calls whose rows have at most two partials each (one prompt-span split and
+// one generated-span split, or fewer): four rows per warp, a quarter-warp per
+// row, so twice the rows per warp are in flight; the same bits as the
+// two-row path.
+template <int D>
+__global__ void __launch_bounds__(256, 3) merge_kernel4(AttnParams P) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    const long warp = (long(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    const long total = long(P.B) * P.Hq;
+    const long row0 = 4 * warp;
+    if (row0 >= total) return;
+    if (merge_rows_group<D, 2, 4>(P, row0, lane)) return;
+    for (long r = row0; r < row0 + 4 && r < total; r += 2)
+        if (!merge_rows_fast2<D, 4>(P, r, lane)) {
+            merge_row(P, r, lane);
+            if (r + 1 < total) merge_row(P, r + 1, lane);
+        }
+}
+
 }  // namespace
 
 int launch_append(const uint16_t* kn, const uint16_t* vn, uint16_t* ks, uint16_t* vs, int B, int N,
@@ -74,7 +94,10 @@ int launch_append(const uint16_t* kn, const uint16_t* vn, uint16_t* ks, uint16_t
 int launch_merge(const AttnParams& p, void* stream, bool overlap_previous) {
     const long rows = long(p.B) * p.Hq;
     const int block = 256;
-    const long warps = p.D <= 128 ? (rows + 1) / 2 : rows;
+    // at most two partials per row: the prompt-span splits (none for a ZERO
+    // row), the generated-span splits and a delta row's splits
+    const bool four = p.D <= 128 && p.nsp + p.nss + (p.delta_on ? p.nsd : 0) <= 2;
+    const long warps = four ? (rows + 3) / 4 : (p.D <= 128 ? (rows + 1) / 2 : rows);
     const long threads = warps * 32;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(unsigned((threads + block - 1) / block));
@@ -85,6 +108,10 @@ int launch_merge(const AttnParams& p, void* stream, bool overlap_previous) {
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = overlap_previous ? 1 : 0;
+    if (four) {
+        if (p.D == 64) return int(cudaLaunchKernelEx(&cfg, merge_kernel4<64>, p));
+        return int(cudaLaunchKernelEx(&cfg, merge_kernel4<128>, p));
+    }
     switch (p.D) {
         case 64: return int(cudaLaunchKernelEx(&cfg, merge_kernel<64>, p));
         case 128: return int(cudaLaunchKernelEx(&cfg, merge_kernel<128>, p));

@@ -108,18 +108,20 @@ __device__ __forceinline__ bool merge_row_fast(const AttnParams& P, long row, in
     return true;
 }
 
-// Two rows per warp, one per half-warp (lanes 0-15 row0, 16-31 row0 + 1),
-// for rows of at most NF live partials each: the loads of both rows go out
-// at once, twice the rows in flight per warp.  The reductions run over the
-// 16 lanes of a half with the partials on lanes 0 .. n-1 of it, so they add
-// the same values in the same order as merge_weights over 32 lanes (the
-// other lanes hold zeros): the same bits as merge_row_fast.  False (nothing
-// written) if either row has more partials.
-template <int D, int NF>
-__device__ __forceinline__ bool merge_rows_fast2(const AttnParams& P, long row0, int lane) {
+// RPW rows per warp (2 or 4), 32 / RPW lanes per row (lanes 0-15 row0,
+// 16-31 row0 + 1 for RPW = 2), for rows of at most NF live partials each:
+// the loads of all the warp's rows go out at once.  The reductions run over
+// the row's lanes with the partials on its first n lanes, so they add the
+// same values in the same order as merge_weights over 32 lanes (the other
+// lanes hold zeros): the same bits as merge_row_fast.  False (nothing
+// written) if any of the rows has more partials.
+template <int D, int NF, int RPW>
+__device__ __forceinline__ bool merge_rows_group(const AttnParams& P, long row0, int lane) {
+    constexpr int LPR = 32 / RPW;                // lanes per row
+    static_assert(NF <= LPR, "a row's partials sit on its first lanes");
     constexpr int C4 = D / 4;                    // float4 slices of a row
-    constexpr int SL = (C4 + 15) / 16;           // slices per lane of a half
-    const int half = lane >> 4, hl = lane & 15;
+    constexpr int SL = (C4 + LPR - 1) / LPR;     // slices per lane
+    const int half = lane / LPR, hl = lane % LPR;
     const long total = long(P.B) * P.Hq;
     const long row = row0 + half;
     const bool live_row = row < total;
@@ -140,20 +142,20 @@ __device__ __forceinline__ bool merge_rows_fast2(const AttnParams& P, long row0,
         const float4* src = reinterpret_cast<const float4*>(P.ws_o + (size_t(merge_slot(i, rp)) * plane + row) * D);
 #pragma unroll
         for (int q = 0; q < SL; ++q) {
-            const int c = hl + 16 * q;
+            const int c = hl + LPR * q;
             ov[i][q] = (i < n && c < C4) ? __ldcg(src + c) : make_float4(0.f, 0.f, 0.f, 0.f);
         }
     }
-    // weights over the half: as merge_weights
+    // weights over the row's lanes: as merge_weights
     const bool zero_span = code == SPLICE_SRC_ZERO && P.p_hi > P.p_lo;
     float M = (hl < n && ml.y > 0.f) ? ml.x : -INFINITY;
     if (zero_span) M = fmaxf(M, 0.f);
 #pragma unroll
-    for (int off = 8; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    for (int off = LPR / 2; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
     const float w = (hl < n && ml.y > 0.f) ? exp2f(ml.x - M) : 0.f;
     float den = w * ml.y;
 #pragma unroll
-    for (int off = 8; off > 0; off >>= 1) den += __shfl_xor_sync(0xffffffffu, den, off);
+    for (int off = LPR / 2; off > 0; off >>= 1) den += __shfl_xor_sync(0xffffffffu, den, off);
     if (zero_span) den = fmaf(float(P.p_hi - P.p_lo), exp2f(0.f - M), den);
     const float inv = den > 0.f ? 1.f / den : 0.f;
     float4 acc[SL];
@@ -161,7 +163,7 @@ __device__ __forceinline__ bool merge_rows_fast2(const AttnParams& P, long row0,
     for (int q = 0; q < SL; ++q) acc[q] = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
     for (int i = 0; i < NF; ++i) {
-        const float wi = __shfl_sync(0xffffffffu, w, (half << 4) + i);
+        const float wi = __shfl_sync(0xffffffffu, w, half * LPR + i);
         if (i < n && wi != 0.f) {
 #pragma unroll
             for (int q = 0; q < SL; ++q) {
@@ -176,11 +178,16 @@ __device__ __forceinline__ bool merge_rows_fast2(const AttnParams& P, long row0,
         float4* out = reinterpret_cast<float4*>(P.out + size_t(row) * D);
 #pragma unroll
         for (int q = 0; q < SL; ++q) {
-            const int c = hl + 16 * q;
+            const int c = hl + LPR * q;
             if (c < C4) out[c] = make_float4(acc[q].x * inv, acc[q].y * inv, acc[q].z * inv, acc[q].w * inv);
         }
     }
     return true;
+}
+
+template <int D, int NF>
+__device__ __forceinline__ bool merge_rows_fast2(const AttnParams& P, long row0, int lane) {
+    return merge_rows_group<D, NF, 2>(P, row0, lane);
 }
 
 // Any number of live partials (up to kMaxSplits): weights first, then the o
