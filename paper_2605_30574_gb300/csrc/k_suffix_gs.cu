@@ -134,7 +134,7 @@ __device__ __forceinline__ void item_of(const AttnParams& P, int idx, Item& it) 
 
 template <int D, int GT>
 __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
-    gs_kernel(const AttnParams P, int n_items) {
+    gs_kernel(const AttnParams P, int n_items, int sm_count) {
     using C = GS<D, GT>;
     extern __shared__ __align__(128) uint8_t smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -171,17 +171,28 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
     }
     __syncwarp();
 
-    // ---- work items: warp w of the grid starts on item w.  As the call's
-    // first pass (all warps start together) it then walks items w + k *
+    // ---- work items: the warp of rank r starts on item r.  As the call's
+    // first pass (all warps start together) it then walks items r + k *
     // (warps of the grid): the extra items of an uneven share land on the
-    // first CTAs, so the other SMs come free whole and early for the
+    // lowest ranks, so the other SMs come free whole and early for the
     // prompt-span pass queued behind.  Behind the prompt-span pass (CTAs
     // start as that pass's CTAs leave) every later item is claimed from the
     // launch-wide counter (numbered from the grid's warp count on), one
     // ahead: lane 0 holds the claim in flight, whose value is needed only
     // when the next item starts ----
     const unsigned nwarps = gridDim.x * C::WARPS;
-    const int first_item = int(blockIdx.x * C::WARPS + warp);
+    // The warps' ranks, SM-major when the grid is whole waves of sm_count
+    // CTAs: the first wave's CTAs land on distinct SMs and each later wave
+    // stacks one more CTA on each in the same order, so CTAs b, b +
+    // sm_count, ... share an SM and get consecutive ranks -- the extra items
+    // of an uneven share then fill whole SMs, and the others come free
+    // together.
+    int rank = int(blockIdx.x) * C::WARPS + warp;
+    if (sm_count > 0 && gridDim.x % unsigned(sm_count) == 0) {
+        const int cps = int(gridDim.x) / sm_count;
+        rank = ((int(blockIdx.x) % sm_count) * cps + int(blockIdx.x) / sm_count) * C::WARPS + warp;
+    }
+    const int first_item = rank;
     const bool claims = P.gs_after_prefix != 0;
     unsigned claim = unsigned(first_item) + nwarps;
     if (claims && lane == 0) claim = nwarps + atomicAdd(P.sched + 2, 1u);
@@ -565,7 +576,7 @@ int launch_gs_t(const AttnParams& p, int n_items, cudaStream_t st, bool overlap_
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = overlap_previous ? 1 : 0;
-    return int(cudaLaunchKernelEx(&cfg, gs_kernel<D, GT>, p, n_items));
+    return int(cudaLaunchKernelEx(&cfg, gs_kernel<D, GT>, p, n_items, sms));
 }
 
 }  // namespace
