@@ -181,14 +181,16 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
     // ahead: lane 0 holds the claim in flight, whose value is needed only
     // when the next item starts ----
     const unsigned nwarps = gridDim.x * C::WARPS;
-    // The warps' ranks, SM-major when the grid is whole waves of sm_count
-    // CTAs: the first wave's CTAs land on distinct SMs and each later wave
-    // stacks one more CTA on each in the same order, so CTAs b, b +
-    // sm_count, ... share an SM and get consecutive ranks -- the extra items
-    // of an uneven share then fill whole SMs, and the others come free
-    // together.
+    // The warps' ranks.  With the prompt-span pass queued behind, SM-major
+    // when the grid is whole waves of sm_count CTAs: the first wave's CTAs
+    // land on distinct SMs and each later wave stacks one more CTA on each
+    // in the same order, so CTAs b, b + sm_count, ... share an SM and get
+    // consecutive ranks -- the extra items of an uneven share then fill
+    // whole SMs, and the others come free together for that pass.  With
+    // nothing queued behind, CTA-major, which spreads the extra items over
+    // the SMs.
     int rank = int(blockIdx.x) * C::WARPS + warp;
-    if (sm_count > 0 && gridDim.x % unsigned(sm_count) == 0) {
+    if (P.prefix_after_gs && sm_count > 0 && gridDim.x % unsigned(sm_count) == 0) {
         const int cps = int(gridDim.x) / sm_count;
         rank = ((int(blockIdx.x) % sm_count) * cps + int(blockIdx.x) / sm_count) * C::WARPS + warp;
     }
