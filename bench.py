@@ -292,15 +292,17 @@ def host_cores():
     return max(1, aff), os.cpu_count() or 1
 
 
-def cpu_baseline(name, budget_s=15.0, batch=0):
+def cpu_baseline(name, budget_s=8.0, batch=0):
+    """The oracle on all affined cores, each process about budget_s of its
+    one-thread work (so 10-30 s of CPU work in all), plus the one-thread rate."""
     from paper_2605_30574_gb300.synth import workloads as W
     wl = W.get(name)
     cores, n_cpu = host_cores()
     units = plan_units(wl, batch, seed=7)
-    # one thread: a few units alone
-    n1, w1 = run_oracle_sample(name, [units[:3]])
+    # one thread: 32 units alone
+    n1, w1 = run_oracle_sample(name, [units[:32]])
     per_unit = w1 / max(n1, 1)
-    upc = int(max(1, min(64, budget_s / per_unit)))
+    upc = int(max(1, min(2048, budget_s / per_unit)))
     need = cores * upc
     take = (units * (need // len(units) + 1))[:need]
     n, wall = run_oracle_sample(name, [take[c::cores] for c in range(cores)])
