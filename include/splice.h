@@ -350,6 +350,18 @@ splice_status splice_debug_source_map(splice_desc* desc, int layer, int step, ui
 splice_status splice_plan_stats(const splice_desc* desc, int layer, int step, int* num_groups,
                                 int* num_tiles, int* prompt_visible, int* suffix_visible);
 
+/*
+ * splice_debug_pass_order -- order of the two attention passes in later
+ * calls on the descriptor: 0 (the default) chosen per call from the plan --
+ * the prompt-span pass first when it holds less than one full 3072-key split
+ * per SM, else the generated-span pass first; 1 the prompt-span pass first;
+ * 2 the generated-span pass first.  Outputs and stores are bit-identical in
+ * every order (the passes write disjoint partial states that the merge
+ * combines in a fixed order); only the overlap of the two passes changes.
+ * SPLICE_EINVAL for another value.  No device work.
+ */
+splice_status splice_debug_pass_order(splice_desc* desc, int order);
+
 /* Synchronise the device and report kernel-side errors recorded since the
  * descriptor was created (SPLICE_EDEVICE), clearing the record. */
 splice_status splice_check_device_error(splice_desc* desc);

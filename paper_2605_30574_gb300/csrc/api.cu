@@ -27,6 +27,7 @@ struct splice_desc {
     Plan plan;
     int device = -1;
     int sms = 0;                        // multiprocessors of the device
+    int pass_order = 0;                 // 0 chosen per call, 1 prompt-span pass first, 2 generated-span pass first
     // Device tables, one allocation.
     char* dev = nullptr;
     std::vector<char> staging;          // host image of `dev`, kept for the async upload
@@ -463,7 +464,9 @@ splice_status attn_common(splice_desc* d, int layer, int step, const splice_bf16
         (long(p.n_span_tiles) * ((p_vis + box - 1) / box) +
          long(p.n_tiles - p.n_span_tiles) * (p.nsd ? (d->delta_max + box - 1) / box : 0)) *
         sh.num_kv_heads * box;
-    const bool prefix_first = prefix_launched && prefix_keys < long(d->sms) * splice::kPrefixSplitKeys;
+    const bool prefix_first =
+        prefix_launched && (d->pass_order == 1 ||
+                            (d->pass_order == 0 && prefix_keys < long(d->sms) * splice::kPrefixSplitKeys));
     p.gs_after_prefix = gs_work && prefix_launched && prefix_first && !d->profiling ? 1 : 0;
     p.prefix_after_gs = gs_work && prefix_launched && !prefix_first && !d->profiling ? 1 : 0;
     auto launch_prefix = [&]() -> splice_status {
@@ -777,6 +780,13 @@ splice_status splice_debug_source_map(splice_desc* d, int layer, int step, uint8
     if (g.err != cudaSuccess) return cuda_fail(g.err, "cudaSetDevice");
     cudaError_t e = cudaMemcpy(host_out, d->d_src + size_t(tab) * d->B, d->B, cudaMemcpyDeviceToHost);
     if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy of the source map");
+    return SPLICE_OK;
+}
+
+splice_status splice_debug_pass_order(splice_desc* d, int order) {
+    if (!d) return fail(SPLICE_EINVAL, "NULL descriptor");
+    if (order < 0 || order > 2) return fail(SPLICE_EINVAL, "pass order %d not in [0, 2]", order);
+    d->pass_order = order;
     return SPLICE_OK;
 }
 

@@ -61,6 +61,7 @@ SIGNATURES = {
     "splice_debug_source_map": (_c_int, [_vp, _c_int, _c_int, ctypes.POINTER(ctypes.c_uint8)]),
     "splice_plan_stats": (_c_int, [_vp, _c_int, _c_int, ctypes.POINTER(_c_int), ctypes.POINTER(_c_int),
                                    ctypes.POINTER(_c_int), ctypes.POINTER(_c_int)]),
+    "splice_debug_pass_order": (_c_int, [_vp, _c_int]),
     "splice_delta_bytes": (ctypes.c_size_t, [_vp]),
     "splice_delta_build": (_c_int, [_vp, _vp, _vp, _vp, _vp, _vp, ctypes.c_size_t, ctypes.c_float,
                                     ctypes.POINTER(ctypes.c_float), _vp]),
@@ -234,6 +235,12 @@ def splice_debug_source_map(desc: Desc, layer, step) -> bytes:
     buf = (ctypes.c_uint8 * desc.num_seqs)()
     _check(lib().splice_debug_source_map(desc.handle, layer, step, buf), "splice_debug_source_map")
     return bytes(buf)
+
+
+def splice_debug_pass_order(desc: Desc, order: int) -> None:
+    """0: order of the two passes chosen per call; 1: prompt-span pass first;
+    2: generated-span pass first."""
+    _check(lib().splice_debug_pass_order(desc.handle, order), "splice_debug_pass_order")
 
 
 def splice_plan_stats(desc: Desc, layer, step) -> dict:

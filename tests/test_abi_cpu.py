@@ -172,3 +172,13 @@ def test_status_strings(lib):
         assert S.splice_status_str(st)
     assert lib.splice_desc_destroy(None) == 0
     assert lib.splice_workspace_bytes(None) == 0
+
+
+def test_pass_order_override_validated(lib):
+    wl = WL.get("tiny")
+    d = _host_desc(wl)
+    for order in (0, 1, 2, 0):
+        S.splice_debug_pass_order(d, order)
+    for bad in (-1, 3):
+        with pytest.raises(S.SpliceError):
+            S.splice_debug_pass_order(d, bad)
