@@ -405,10 +405,19 @@ def profile_pass(sb, steps, qs, kn, vn, outs, run_step, stream):
 
 
 def kernel_table(prof, per_kind):
+    """Per kernel kind: launches, summed time, share of the serialised step,
+    algorithmic GB/s, algorithmic bytes per launch and -- where an ncu capture
+    gave the kernel's DRAM bytes per algorithmic byte -- DRAM bytes per launch."""
     total = sum(x[1] for x in prof.values()) or 1.0
-    return {k: {"launches": v[0], "ms_total": round(v[1], 3), "share": round(v[1] / total, 4),
-                "GBps": round(per_kind[k] / (v[1] / 1000.0) / 1e9, 1) if v[1] > 0 else None}
-            for k, v in prof.items()}
+    out = {}
+    for k, v in prof.items():
+        per_launch = per_kind[k] // max(v[0], 1)
+        ratio = TRAFFIC_PER_ALGORITHMIC_BYTE.get(k)
+        out[k] = {"launches": v[0], "ms_total": round(v[1], 3), "share": round(v[1] / total, 4),
+                  "GBps": round(per_kind[k] / (v[1] / 1000.0) / 1e9, 1) if v[1] > 0 else None,
+                  "bytes_per_launch": per_launch,
+                  "traffic_per_launch": round(ratio * per_launch) if ratio and v[0] else None}
+    return out
 
 
 def step_bytes(sb, steps, fused):
