@@ -106,7 +106,12 @@ __device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&v)[8])
 __device__ __forceinline__ void store_p(uint32_t taddr, const uint32_t (&v)[16]) { tmem_st16(taddr, v); }
 __device__ __forceinline__ void store_p(uint32_t taddr, const uint32_t (&v)[8]) { tmem_st8(taddr, v); }
 
-template <int D>
+// SHORT: every item of the launch has at most four key blocks (prompt spans
+// of up to 512 keys at d <= 128).  A V block then waits only briefly for its
+// P V, so V takes the two-stage ring of K and the smem goes to a second Q
+// buffer: the next item's queries are gathered while this item runs, instead
+// of after its last Q K^T.
+template <int D, bool SHORT = false>
 struct Cfg {
     static constexpr int BN = D == 256 ? 64 : 128;          // keys per K/V block
     static constexpr int KPT = BN / 2;                      // keys per softmax thread per block
@@ -117,7 +122,7 @@ struct Cfg {
     // blocks later, so V gets the deeper ring: 192 KB of Q, K and V stages.
     static constexpr uint32_t Q_BYTES = kRows * D * 2;      // Q of one tile
     static constexpr int KST = int((64u * 1024u) / KV_BYTES);      // K stages: 64 KB
-    static constexpr int VST = D == 256 ? KST : KST + KST / 2;     // V stages: 96 KB where smem allows
+    static constexpr int VST = (D == 256 || SHORT) ? KST : KST + KST / 2;   // V stages: 96 KB where smem allows
     static constexpr int NQ = (2 * Q_BYTES + (KST + VST) * KV_BYTES <= 192u * 1024u) ? 2 : 1;   // Q buffers
     // TMEM columns: NSLOT slots of BN columns for S (each softmax thread's
     // P over the first columns of its half of the slot), then O.
@@ -227,13 +232,13 @@ __device__ __forceinline__ ItemInfo item_info(const AttnParams& P, const TcParam
     return it;
 }
 
-template <int D>
+template <int D, bool SHORT>
 __global__ void __launch_bounds__(kThreads, 1)
     prefix_tc_kernel(const __grid_constant__ CUtensorMap tm_kc, const __grid_constant__ CUtensorMap tm_vc,
                      const __grid_constant__ CUtensorMap tm_kd, const __grid_constant__ CUtensorMap tm_vd,
                      const __grid_constant__ CUtensorMap tm_kx, const __grid_constant__ CUtensorMap tm_vx,
                      const TcParams tp) {
-    using C = Cfg<D>;
+    using C = Cfg<D, SHORT>;
     using Bb = Bars<C::KST, C::VST, C::NSLOT>;
     constexpr int NSLOT = C::NSLOT;
     const AttnParams& P = tp.a;
@@ -879,18 +884,19 @@ EncodeFn encode_fn() {
     return fn;
 }
 
-template <int D>
+template <int D, bool SHORT>
 int launch_d(const TcParams& tp, const CUtensorMap* m, cudaStream_t st, bool overlap_previous) {
+    using C = Cfg<D, SHORT>;
     static int sms = 0;
     if (!sms) {
-        cudaFuncSetAttribute(prefix_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<D>::SMEM);
+        cudaFuncSetAttribute(prefix_tc_kernel<D, SHORT>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
         int dev = 0;
         cudaGetDevice(&dev);
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     }
     const unsigned grid = unsigned(tp.n_items < sms ? tp.n_items : sms);
     if (!overlap_previous) {
-        prefix_tc_kernel<D><<<grid, kThreads, Cfg<D>::SMEM, st>>>(m[0], m[1], m[2], m[3], m[4], m[5], tp);
+        prefix_tc_kernel<D, SHORT><<<grid, kThreads, C::SMEM, st>>>(m[0], m[1], m[2], m[3], m[4], m[5], tp);
         return 0;
     }
     // programmatic dependent launch: CTAs may start as the previous grid's
@@ -898,14 +904,14 @@ int launch_d(const TcParams& tp, const CUtensorMap* m, cudaStream_t st, bool ove
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = Cfg<D>::SMEM;
+    cfg.dynamicSmemBytes = C::SMEM;
     cfg.stream = st;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return int(cudaLaunchKernelEx(&cfg, prefix_tc_kernel<D>, m[0], m[1], m[2], m[3], m[4], m[5], tp));
+    return int(cudaLaunchKernelEx(&cfg, prefix_tc_kernel<D, SHORT>, m[0], m[1], m[2], m[3], m[4], m[5], tp));
 }
 
 }  // namespace
@@ -971,10 +977,19 @@ int launch_prefix_tc(const AttnParams& p, const void* maps, const int* bounds, i
     if (tp.n_items <= 0) return 0;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     int r = int(cudaErrorInvalidValue);
+    // every item of at most four key blocks: the short-item ring layout
+    const int bn = prefix_tc_box_rows(p.D);
+    const bool short_items = p.D <= 128 && bounds[1] <= 4 * bn && (p.nsd == 0 || delta_keys <= 4 * bn);
     switch (p.D) {
-        case 64: r = launch_d<64>(tp, m, st, overlap_previous); break;
-        case 128: r = launch_d<128>(tp, m, st, overlap_previous); break;
-        case 256: r = launch_d<256>(tp, m, st, overlap_previous); break;
+        case 64:
+            r = short_items ? launch_d<64, true>(tp, m, st, overlap_previous)
+                            : launch_d<64, false>(tp, m, st, overlap_previous);
+            break;
+        case 128:
+            r = short_items ? launch_d<128, true>(tp, m, st, overlap_previous)
+                            : launch_d<128, false>(tp, m, st, overlap_previous);
+            break;
+        case 256: r = launch_d<256, false>(tp, m, st, overlap_previous); break;
         default: break;
     }
     if (r != 0) return r;
