@@ -59,7 +59,7 @@ NOMINAL_HBM_GBS = 8000.0
 # reduced ladder case (read + written bytes / algorithmic bytes of that launch);
 # traffic grows in proportion to the units a launch processes.  Only kernels
 # whose current build was captured are listed.
-TRAFFIC_PER_ALGORITHMIC_BYTE = {"generated_span_pass": (539.054 + 6.104) / 541.065,
+TRAFFIC_PER_ALGORITHMIC_BYTE = {"generated_span_pass": (539.065 + 6.550) / 541.065,
                                 "prompt_span_pass": (236.987 + 2.962) / 234.881}
 
 
