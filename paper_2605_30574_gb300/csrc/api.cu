@@ -448,12 +448,12 @@ splice_status attn_common(splice_desc* d, int layer, int step, const splice_bf16
     // the first pass's CTAs leave, and it waits for the first pass before it
     // exits; the merge is queued behind the second pass.  So the first pass's
     // tail is filled and the second pass's is not.  The generated-span pass
-    // goes first when the prompt-span pass holds at least one full split
-    // (kPrefixSplitKeys keys) per SM: then the prompt-span pass's items fill
-    // the generated-span pass's tail.  A smaller prompt-span pass goes first:
-    // its short run and its tail (part of the SMs idle while its last items
-    // finish) are filled by the generated-span pass's run-time claimed
-    // units.  With per-launch timing on, the events between the launches
+    // goes first when the prompt-span pass holds at least
+    // kPrefixFirstKeysPerSm keys per SM: then the prompt-span pass's items
+    // fill the generated-span pass's tail.  A smaller prompt-span pass goes
+    // first: its short run and its tail (part of the SMs idle while its last
+    // items finish) are filled by the generated-span pass's run-time claimed
+    // items.  With per-launch timing on, the events between the launches
     // serialise everything.
     const bool gs_work = p.nss > 0;
     const long prefix_items = long(p.n_span_tiles) * sh.num_kv_heads * p.nsp +
@@ -466,7 +466,7 @@ splice_status attn_common(splice_desc* d, int layer, int step, const splice_bf16
         sh.num_kv_heads * box;
     const bool prefix_first =
         prefix_launched && (d->pass_order == 1 ||
-                            (d->pass_order == 0 && prefix_keys < long(d->sms) * splice::kPrefixSplitKeys));
+                            (d->pass_order == 0 && prefix_keys < long(d->sms) * splice::kPrefixFirstKeysPerSm));
     p.gs_after_prefix = gs_work && prefix_launched && prefix_first && !d->profiling ? 1 : 0;
     p.prefix_after_gs = gs_work && prefix_launched && !prefix_first && !d->profiling ? 1 : 0;
     auto launch_prefix = [&]() -> splice_status {

@@ -939,23 +939,25 @@ int prefix_tc_splits(int d, int p_vis, int max_splits, int* bounds) {
     // Splits depend only on the visible span length (and the cap), so a
     // row's arithmetic never depends on which other rows share its tile or
     // launch.  Every item gathers its tile's queries and stores its partial
-    // states, so fewer, longer items move fewer bytes: splits of kPrefixSplitKeys
-    // keys, all but the last full.  A longer span ends in a shorter split,
-    // which the split-major item order hands out last, so a launch ends on
-    // short items.  Past the cap, the blocks are shared out evenly.
+    // states, so long items move fewer bytes; but a launch ends as unevenly
+    // as its last items are long.  So a span's first split is
+    // kPrefixFirstSplitKeys keys and the rest kPrefixSplitKeys: the
+    // split-major item order hands out every span's long first split before
+    // the short ones, and the launch ends on short items.  Past the cap, the
+    // blocks are shared out evenly.
     const int bn = prefix_tc_box_rows(d);
     const int nb = (p_vis + bn - 1) / bn;
-    const int full = kPrefixSplitKeys / bn;
-    int ns = (nb + full - 1) / full;
+    const int first = kPrefixFirstSplitKeys / bn, rest = kPrefixSplitKeys / bn;
+    const int ns_full = nb <= first ? 1 : 1 + (nb - first + rest - 1) / rest;
     bounds[0] = 0;
-    if (ns <= max_splits) {
-        for (int i = 0; i < ns; ++i) {
-            const int b = bounds[i] + full * bn;
+    if (ns_full <= max_splits) {
+        for (int i = 0; i < ns_full; ++i) {
+            const int b = bounds[i] + (i == 0 ? first : rest) * bn;
             bounds[i + 1] = b < p_vis ? b : p_vis;
         }
-        return ns;
+        return ns_full;
     }
-    ns = max_splits;
+    const int ns = max_splits;
     for (int i = 0; i < ns; ++i) {
         const int blocks = nb / ns + (i < nb % ns ? 1 : 0);
         const int b = bounds[i] + blocks * bn;

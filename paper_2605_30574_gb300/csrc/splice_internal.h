@@ -20,8 +20,13 @@ constexpr int kMaxSuffixSplits = 8;
 constexpr int kMaxSplits = kMaxPrefixSplits + kMaxSuffixSplits;
 // Rows of one tensor-core prefix tile (tcgen05 M).
 constexpr int kTileRows = 128;
-// Keys of a full prompt-span split (every split of a span but its last).
-constexpr int kPrefixSplitKeys = 3072;
+// Prompt-span splits: a span's first split holds kPrefixFirstSplitKeys keys,
+// every later one kPrefixSplitKeys (the last possibly fewer).
+constexpr int kPrefixFirstSplitKeys = 2048;
+constexpr int kPrefixSplitKeys = 1024;
+// The call's prompt-span pass goes first when it holds fewer than this many
+// keys (summed over its items) per SM.
+constexpr int kPrefixFirstKeysPerSm = 3072;
 // Group source flag: the group reads the delta-encoded rows of a donor slot
 // (group_src = kGroupDelta | (SPLICE_SRC_DONOR0 + slot)).
 constexpr int32_t kGroupDelta = SPLICE_GROUP_DELTA;
