@@ -339,13 +339,21 @@ def reference_arm(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * total_wall / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic",
-            "config": {"workload": describe(wl), "batch": wl.batch},
+            "config": workload_config(wl, args.batch, args.gpus),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "os_cpu_count": n_cpu, "kind": "oracle",
                              "sample": f"each step: {cores} (sequence, layer, step) units of batch {args.batch} "
                                        f"from the parity sampling plan, one per core; input generation excluded"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
     return 0
+
+
+def workload_config(wl, batch: int, world: int) -> dict:
+    """The `config` of both arms' lines: the workload, its batch, the layout
+    over GPUs (identical for the same workload, whatever runs it)."""
+    lo, hi = wl.batch_range(batch)
+    return {"workload": describe(wl), "batch": f"batch {batch} of {wl.num_batches()}: sequences {lo}-{hi - 1}",
+            "parallelism": f"{world} GPU(s), one sweep batch each, no collective"}
 
 
 def describe(wl):
@@ -525,12 +533,10 @@ def gpu_arm(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": len(steps),
             "warmup": args.warmup, "ms_per_step": ms / len(steps), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": describe(wl), "batch": f"batch {batch} of {wl.num_batches()}: sequences "
-                                                           f"{wl.batch_range(batch)[0]}-{wl.batch_range(batch)[1] - 1}",
-                       "call": "spliced_decode_step (append fused into the generated-span pass)" if fused
-                               else "suffix_kv_append + spliced_decode_attn",
-                       "decode_steps_t": steps, "l2": "inputs larger than L2 (every step streams >10 GB); no flush",
-                       "parallelism": f"{world} GPU(s), one sweep batch each, no collective"},
+            "config": workload_config(wl, batch, world),
+            "call": "spliced_decode_step (append fused into the generated-span pass)" if fused
+                    else "suffix_kv_append + spliced_decode_attn",
+            "decode_steps_t": steps, "l2": "inputs larger than L2 (every step streams >10 GB); no flush",
             "hbm": {"algorithmic_GB_per_step": round(total_bytes / len(steps) / 1e9, 3),
                     "achieved_GBps": round(total_bytes / (ms / 1000.0) / 1e9, 1),
                     "frac_of_measured": round(total_bytes / (ms / 1000.0) / 1e9 / peak, 4),
