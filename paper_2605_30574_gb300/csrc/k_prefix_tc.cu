@@ -102,6 +102,13 @@ __device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&v)[8])
                  : "memory");
 }
 
+// 8 floats to global memory in one 256-bit store (32-byte aligned address).
+__device__ __forceinline__ void st_global_v8(float* p, const float* v) {
+    asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "f"(v[0]), "f"(v[1]),
+                 "f"(v[2]), "f"(v[3]), "f"(v[4]), "f"(v[5]), "f"(v[6]), "f"(v[7])
+                 : "memory");
+}
+
 // One segment's P (bf16 pairs), by segment size.
 __device__ __forceinline__ void store_p(uint32_t taddr, const uint32_t (&v)[16]) { tmem_st16(taddr, v); }
 __device__ __forceinline__ void store_p(uint32_t taddr, const uint32_t (&v)[8]) { tmem_st8(taddr, v); }
@@ -812,9 +819,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         tc::tmem_wait_ld();
                         if (valid) {
 #pragma unroll
-                            for (int i = 0; i < 32; i += 4)
-                                *reinterpret_cast<float4*>(op + q * 32 + i) =
-                                    make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+                            for (int i = 0; i < 32; i += 8) st_global_v8(op + q * 32 + i, v + i);
                         }
                     }
                 }
