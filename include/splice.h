@@ -177,7 +177,9 @@ splice_status suffix_kv_append(splice_desc* desc, int layer, int step, const spl
  *   k_donor, v_donor    donor store (layout above); may be NULL when no slot is stored
  *   k_suffix, v_suffix  generated-span store, slots 0 .. step-1 valid
  *   out                 [num_seqs][Hq][d] fp32, softmax(sm_scale q K^T) V per q head
- *   workspace           device scratch of at least splice_workspace_bytes(desc) bytes
+ *   workspace           device scratch of at least splice_workspace_bytes(desc) bytes,
+ *                       16-byte aligned (the library places its arrays on 256-byte
+ *                       boundaries inside it; the size includes that slack)
  *
  * 0 <= layer < N, 0 <= step <= max_steps (step 0 = empty generated span, a
  * degenerate case for tests; a row with no visible key outputs 0).

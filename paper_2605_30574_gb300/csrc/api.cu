@@ -318,11 +318,14 @@ cudaError_t timed_launch(splice_desc* d, int kind, void* stream, F&& launch) {
     return e;
 }
 
+// The workspace: (m, l) of every partial state, then o, each part starting
+// on a 256-byte boundary whatever the alignment of the caller's pointer (the
+// kernels store o with 32-byte vector stores), hence the 256 bytes of slack.
 size_t workspace_bytes_of(const splice_desc* d) {
     const size_t rows = size_t(d->B) * d->shape.num_q_heads;
     const size_t ml = align_up(size_t(splice::kMaxSplits) * rows * sizeof(float2), 256);
     const size_t o = size_t(splice::kMaxSplits) * rows * d->shape.head_dim * sizeof(float);
-    return ml + o;
+    return 256 + ml + o;
 }
 
 // One attention call: validation, the (epoch, layer class) table of (layer,
@@ -370,9 +373,9 @@ splice_status attn_common(splice_desc* d, int layer, int step, const splice_bf16
     p.vs_w = v_suffix;
     p.fuse_append = k_new ? 1 : 0;
     p.out = out;
-    p.ws_ml = static_cast<float2*>(workspace);
-    p.ws_o = reinterpret_cast<float*>(static_cast<char*>(workspace) +
-                                      align_up(size_t(splice::kMaxSplits) * rows * sizeof(float2), 256));
+    char* ws_base = reinterpret_cast<char*>(align_up(reinterpret_cast<uintptr_t>(workspace), 256));
+    p.ws_ml = reinterpret_cast<float2*>(ws_base);
+    p.ws_o = reinterpret_cast<float*>(ws_base + align_up(size_t(splice::kMaxSplits) * rows * sizeof(float2), 256));
     p.src = d->d_src + size_t(tab) * d->B;
     p.seq_prompt = d->d_seq_prompt;
     p.seq_slot = d->d_seq_slot;

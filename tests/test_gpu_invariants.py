@@ -164,6 +164,25 @@ def test_argument_errors_on_device_descriptor():
     S.splice_check_device_error(a.desc)
 
 
+def test_workspace_alignment_does_not_change_results():
+    """The workspace need only be 16-byte aligned: the library places its
+    partial-state arrays on 256-byte boundaries inside it, so an offset
+    pointer gives the same bits."""
+    wl = small_wl()
+    a = SweepBatch(wl, seqs=wl.sequences())
+    nbytes = S.splice_workspace_bytes(a.desc)
+    big = torch.empty(nbytes + 256, dtype=torch.uint8, device="cuda")
+    for l, t in ((0, 1), (3, 5), (1, 12)):
+        ref = a.run(l, t).clone()
+        for off in (16, 48, 240):
+            a.out.fill_(float("nan"))
+            S.spliced_decode_attn(a.desc, l, t, a.q, a.k_clean, a.v_clean, a.k_donor, a.v_donor,
+                                  a.k_suffix, a.v_suffix, a.out, big.data_ptr() + off, workspace_bytes=nbytes)
+            torch.cuda.synchronize()
+            assert torch.equal(a.out, ref), (l, t, off)
+    S.splice_check_device_error(a.desc)
+
+
 def test_bounded_wait_reports_instead_of_hanging():
     """A wait that can never complete gives up after its limit and the host
     reads SPLICE_EDEVICE; the context stays usable and the record clears."""
