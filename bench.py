@@ -60,7 +60,7 @@ NOMINAL_HBM_GBS = 8000.0
 # traffic grows in proportion to the units a launch processes.  Only kernels
 # whose current build was captured are listed.
 TRAFFIC_PER_ALGORITHMIC_BYTE = {"generated_span_pass": (539.065 + 6.550) / 541.065,
-                                "prompt_span_pass": (240.985 + 5.274) / 234.881}
+                                "prompt_span_pass": (237.003 + 4.812) / 234.881}
 
 
 def step_schedule(T: int, n: int, offset: int = 0):
