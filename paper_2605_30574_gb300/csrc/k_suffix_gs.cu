@@ -96,9 +96,9 @@ struct GS {
     static constexpr uint32_t OFF_RED = 2 * STAGE;
     static constexpr uint32_t OFF_PP = OFF_RED + KPW * GSTRIDE * 4;
     static constexpr uint32_t OFF_BAR = OFF_PP + KPW * NV * 8;
-    static constexpr uint32_t OFF_TAKEN = OFF_BAR + 16;       // [4] items in the order the issue cursor took them
+    static constexpr uint32_t OFF_TAKEN = OFF_BAR + 16;       // [4] items (decoded) in the order the issue cursor took them
     static constexpr uint32_t QROWS = GT * D * 2;             // the GT query rows of one item
-    static constexpr uint32_t OFF_Q = OFF_TAKEN + 16;         // [2] query rows, brought with each item's first block
+    static constexpr uint32_t OFF_Q = OFF_TAKEN + 4 * 32;     // [2] query rows, brought with each item's first block
     static constexpr uint32_t PER_WARP = (OFF_Q + 2 * QROWS + 127) / 128 * 128;
     static constexpr uint32_t SMEM = WARPS * PER_WARP;
     static_assert(NV % 4 == 0 || NV < 4, "reduce layout");
@@ -106,30 +106,51 @@ struct GS {
     static_assert(LPK % GT == 0, "the logits of a lane belong to one query row");
 };
 
-// Where the keys of one work item live.
+// n / d for 0 <= n < 2^31 by a multiply and a shift, for a divisor fixed
+// per launch (Granlund and Montgomery, "Division by invariant integers using
+// multiplication", 1994, the round-up method): with s = ceil(log2 d) and
+// m = floor(2^32 (2^s - d) / d) + 1, n / d = (umulhi(n, m) + n) >> s; the
+// sum stays below 2^32 because umulhi(n, m) < n < 2^31.
+struct FastDiv {
+    uint32_t d, m, s;
+    __device__ explicit FastDiv(int divisor) : d(uint32_t(divisor)), m(1), s(0) {
+        while ((1u << s) < d) ++s;
+        m = uint32_t((((uint64_t(1) << s) - d) << 32) / d + 1);
+    }
+    __device__ __forceinline__ int div(int n) const { return int((__umulhi(uint32_t(n), m) + uint32_t(n)) >> s); }
+};
+
+struct ItemDivs {
+    FastDiv nss, n_rc, hkv;
+};
+
+// One work item: where its rows and keys are.  The issue cursor decodes
+// each item once and hands it to the consumer through the warp's ring
+// (eight ints, idx -1 for the end of the walk).
 struct Item {
-    const uint16_t* k;
-    const uint16_t* v;
-    int s, h, rc, split, k0, k1, nblk;
+    int idx, s, h, rc, split, k0, k1, nblk;
 };
 
 // Work item idx = ((sequence * Hkv + kv head) * row chunks + row chunk) *
 // splits + key split.
-template <int D, int GT>
-__device__ __forceinline__ void item_of(const AttnParams& P, int idx, Item& it) {
-    const int n_rc = P.G / GT;
-    it.split = idx % P.nss;
-    int rem = idx / P.nss;
-    it.rc = rem % n_rc;
-    rem /= n_rc;
-    it.h = rem % P.Hkv;
-    it.s = rem / P.Hkv;
-    const size_t blk = ((size_t(it.s) * P.N + P.layer) * P.Hkv + it.h) * size_t(P.T);
-    it.k = P.ks + blk * D;
-    it.v = P.vs + blk * D;
+__device__ __forceinline__ void item_of(const AttnParams& P, const ItemDivs& dv, int idx, Item& it) {
+    it.idx = idx;
+    int rem = dv.nss.div(idx);
+    it.split = idx - rem * P.nss;
+    const int sh = dv.n_rc.div(rem);
+    it.rc = rem - sh * int(dv.n_rc.d);
+    it.s = dv.hkv.div(sh);
+    it.h = sh - it.s * P.Hkv;
     it.k0 = P.s_lo + it.split * P.s_chunk;
     it.k1 = min(P.s_hi, it.k0 + P.s_chunk);
     it.nblk = it.k1 > it.k0 ? (it.k1 - it.k0 + 15) / 16 : 0;
+}
+
+// Offset (in elements) of the generated-span K/V rows of (sequence, kv head)
+// at this layer.
+template <int D>
+__device__ __forceinline__ size_t span_base(const AttnParams& P, int s, int h) {
+    return ((size_t(s) * P.N + P.layer) * P.Hkv + h) * size_t(P.T) * D;
 }
 
 template <int D, int GT>
@@ -157,7 +178,7 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
     const uint32_t bar0 = wbase + C::OFF_BAR;
     float* red = reinterpret_cast<float*>(ws + C::OFF_RED);
     float2* pp = reinterpret_cast<float2*>(ws + C::OFF_PP);
-    int* taken_items = reinterpret_cast<int*>(ws + C::OFF_TAKEN);
+    int4* ring = reinterpret_cast<int4*>(ws + C::OFF_TAKEN);
 
     const int gi = lane / C::LPK, dl = lane % C::LPK;
     const int g_mine = dl % GT;
@@ -210,29 +231,38 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
     };
 
     // ---- issue cursor: walks (item, block) in claim order and records every
-    // item it takes (then -1) for the consumer.  It runs two blocks ahead and
-    // every item has a block (the host keeps at least 64 keys per split), so
-    // it is at most two items ahead ----
+    // item it takes, decoded (then the end, idx -1), for the consumer.  It
+    // runs two blocks ahead and every item has a block (the host keeps at
+    // least 64 keys per split), so it is at most two items ahead ----
+    const ItemDivs dv{FastDiv(P.nss), FastDiv(P.G / GT), FastDiv(P.Hkv)};
     Item iss;
-    int iss_idx = first_item < n_items ? first_item : -1, iss_b = 0, recorded = 1;
-    if (lane == 0) taken_items[0] = iss_idx;
+    int iss_idx = first_item < n_items ? first_item : -1, iss_b = 0, recorded = 0;
     bool iss_ok = false;
+    auto record = [&](const Item& e) {
+        if (lane == 0) {
+            ring[2 * (recorded & 3)] = make_int4(e.idx, e.s, e.h, e.rc);
+            ring[2 * (recorded & 3) + 1] = make_int4(e.split, e.k0, e.k1, e.nblk);
+        }
+        ++recorded;
+    };
     auto seek = [&]() {   // the first block at or after item iss_idx
         iss_ok = false;
         while (iss_idx >= 0) {
-            item_of<D, GT>(P, iss_idx, iss);
+            item_of(P, dv, iss_idx, iss);
+            record(iss);
             if (iss.nblk > 0) {
                 iss_ok = true;
                 return;
             }
             iss_idx = next_item();
-            if (lane == 0) taken_items[recorded & 3] = iss_idx;
-            ++recorded;
         }
+        iss.idx = -1;
+        record(iss);
     };
     seek();
     int issued = 0, iss_items = 0;
     const uint64_t pol = l2_evict_first_policy();
+    size_t iss_base = iss_ok ? span_base<D>(P, iss.s, iss.h) : 0;
     auto issue_next = [&]() {
         if (!iss_ok) return;
         const int stg = issued & 1;
@@ -252,8 +282,8 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
                 bulk_copy_plain(wbase + C::OFF_Q + (iss_items & 1) * C::QROWS,
                                 P.q + (size_t(iss.s) * P.Hq + iss.h * P.G + iss.rc * GT) * D, C::QROWS, bar0 + 8 * stg);
             if (bytes) {
-                bulk_copy(dst, iss.k + size_t(j) * D, bytes, bar0 + 8 * stg, pol);
-                bulk_copy(dst + C::BK * C::ROW, iss.v + size_t(j) * D, bytes, bar0 + 8 * stg, pol);
+                bulk_copy(dst, P.ks + iss_base + size_t(j) * D, bytes, bar0 + 8 * stg, pol);
+                bulk_copy(dst + C::BK * C::ROW, P.vs + iss_base + size_t(j) * D, bytes, bar0 + 8 * stg, pol);
             }
         }
         ++issued;
@@ -261,9 +291,8 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
         if (++iss_b >= iss.nblk) {
             iss_b = 0;
             iss_idx = next_item();
-            if (lane == 0) taken_items[recorded & 3] = iss_idx;
-            ++recorded;
             seek();
+            if (iss_ok) iss_base = span_base<D>(P, iss.s, iss.h);
         }
     };
     issue_next();
@@ -273,10 +302,10 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
     bool ok = true;
     for (int taken = 0; ok; ++taken) {
         __syncwarp();
-        const int idx = taken_items[taken & 3];
-        if (idx < 0) break;
-        Item it;
-        item_of<D, GT>(P, idx, it);
+        const int4 e0 = ring[2 * (taken & 3)];
+        if (e0.x < 0) break;
+        const int4 e1 = ring[2 * (taken & 3) + 1];
+        const Item it{e0.x, e0.y, e0.z, e0.w, e1.x, e1.y, e1.z, e1.w};
         // q rows of this item, pre-scaled into log2 units, as dim pairs: in
         // the item's query buffer once its first block has landed
         float2 q2[GT][8];
@@ -486,9 +515,26 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
             l[g] = x;
         }
 
-        // ---- combine the KPW key groups of the warp, write the partial ----
+        // ---- combine the KPW key groups of the warp, a reduce-scatter: round
+        // r pairs group gi with group gi ^ 2^r, both rescale to the pair's
+        // max, and each keeps the half of its dims that its partner sends
+        // it; after log2(KPW) rounds every lane holds F = 16 / KPW dims of
+        // every row, summed over the groups, and m, l of every row ----
+        constexpr int F = 16 / C::KPW;
+        float v[GT][16];
 #pragma unroll
-        for (int off = C::LPK; off < 32; off <<= 1) {
+        for (int g = 0; g < GT; ++g) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                v[g][2 * i] = o2[g][i].x;
+                v[g][2 * i + 1] = o2[g][i].y;
+            }
+        }
+        int kept = 0;   // first of this lane's dims, as an index into its 16
+#pragma unroll
+        for (int r = 0; (C::LPK << r) < 32; ++r) {
+            const int off = C::LPK << r, W = 16 >> r;
+            const bool hi = (gi >> r) & 1;
 #pragma unroll
             for (int g = 0; g < GT; ++g) {
                 const float mo = __shfl_xor_sync(kFull, m[g], off);
@@ -498,26 +544,33 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
                 const float bb = mo == -INFINITY ? 0.f : ex2(mo - M);
                 l[g] = l[g] * a + lo * bb;
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const float ox = __shfl_xor_sync(kFull, o2[g][i].x, off);
-                    const float oy = __shfl_xor_sync(kFull, o2[g][i].y, off);
-                    o2[g][i] = make_float2(o2[g][i].x * a + ox * bb, o2[g][i].y * a + oy * bb);
+                for (int k = 0; k < W / 2; ++k) {
+                    const float send = hi ? v[g][k] : v[g][W / 2 + k];
+                    const float keep = hi ? v[g][W / 2 + k] : v[g][k];
+                    const float recv = __shfl_xor_sync(kFull, send, off);
+                    v[g][k] = keep * a + recv * bb;
                 }
                 m[g] = M;
             }
+            if (hi) kept += W / 2;
         }
-        if (gi == 0) {
+        {
             const int slot = kMaxPrefixSplits + it.split;
+            // dims 8 c0 .. 8 c0 + 7 are this lane's first 8, 8 c1 .. its last 8
+            const int dim0 = kept < 8 ? 8 * c0 + kept : 8 * c1 + (kept - 8);
 #pragma unroll
             for (int g = 0; g < GT; ++g) {
                 const size_t row = size_t(it.s) * P.Hq + it.h * P.G + it.rc * GT + g;
                 const size_t idx2 = size_t(slot) * P.B * P.Hq + row;
-                float4* op = reinterpret_cast<float4*>(P.ws_o + idx2 * D);
-                op[2 * c0] = make_float4(o2[g][0].x, o2[g][0].y, o2[g][1].x, o2[g][1].y);
-                op[2 * c0 + 1] = make_float4(o2[g][2].x, o2[g][2].y, o2[g][3].x, o2[g][3].y);
-                op[2 * c1] = make_float4(o2[g][4].x, o2[g][4].y, o2[g][5].x, o2[g][5].y);
-                op[2 * c1 + 1] = make_float4(o2[g][6].x, o2[g][6].y, o2[g][7].x, o2[g][7].y);
-                if (dl == 0) P.ws_ml[idx2] = make_float2(m[g], l[g]);
+                float* op = P.ws_o + idx2 * D + dim0;
+                if constexpr (F == 2) {
+                    *reinterpret_cast<float2*>(op) = make_float2(v[g][0], v[g][1]);
+                } else {
+#pragma unroll
+                    for (int k = 0; k < F; k += 4)
+                        *reinterpret_cast<float4*>(op + k) = make_float4(v[g][k], v[g][k + 1], v[g][k + 2], v[g][k + 3]);
+                }
+                if (lane == 0) P.ws_ml[idx2] = make_float2(m[g], l[g]);
             }
         }
     }
