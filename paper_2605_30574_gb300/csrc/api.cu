@@ -42,7 +42,7 @@ struct splice_desc {
     int32_t* d_group_mask = nullptr;
     int32_t* d_slot_delta = nullptr;
     unsigned* d_err = nullptr;
-    unsigned* d_sched = nullptr;   // [4] work counter and finished-CTA count of each pass (zero between launches)
+    unsigned* d_sched = nullptr;   // [8] work counters, finished counts and the completion flag of the passes
     // Measurement: launch counter and optional per-launch event timing.
     long long launches = 0;
     bool profiling = false;
@@ -192,7 +192,7 @@ splice_status upload_tables(splice_desc* d, void* stream) {
     }
     for (int k = 0; k < d->Dslots; ++k) slot_delta[k] = d->slot_delta[k] ? 1 : 0;
     const unsigned zero = 0;
-    const unsigned sched_zero[4] = {0, 0, 0, 0};
+    const unsigned sched_zero[8] = {0, 0, 0, 0, 0, 0, 0, 0};
     Part parts[] = {
         {pl.src.data(), pl.src.size(), 0},
         {seq_prompt.data(), seq_prompt.size() * 4, 0},
@@ -472,6 +472,16 @@ splice_status attn_common(splice_desc* d, int layer, int step, const splice_bf16
                             (d->pass_order == 0 && prefix_keys < long(d->sms) * splice::kPrefixFirstKeysPerSm));
     p.gs_after_prefix = gs_work && prefix_launched && prefix_first && !d->profiling ? 1 : 0;
     p.prefix_after_gs = gs_work && prefix_launched && !prefix_first && !d->profiling ? 1 : 0;
+    // Behind the prompt-span pass, with one prompt-span and one
+    // generated-span split per row and no delta rows, the generated-span
+    // pass merges each item's rows itself -- ZERO rows always, the others
+    // once the prompt-span pass has completed (a flag it reads without
+    // waiting) -- writes the output and marks the row; the merge kernel
+    // then only merges the rows left unmarked.
+    p.gs_merge = p.gs_after_prefix && p.nss == 1 && p.nsp == 1 && !p.delta_on &&
+                         splice::generated_span_can_merge(sh.head_dim, p.G)
+                     ? 1
+                     : 0;
     auto launch_prefix = [&]() -> splice_status {
         // Tensor maps over the stores viewed as [rows][d]; the delta rows
         // have the donor store's layout.

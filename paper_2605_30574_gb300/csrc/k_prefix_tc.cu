@@ -313,12 +313,23 @@ __global__ void __launch_bounds__(kThreads, 1)
     // work has finished, so it waits for it (its writes visible) before
     // reading anything -- the queries, the work counter, the tables.  Only
     // then may the generated-span pass queued behind this grid launch: it
-    // reads nothing this grid writes, so its CTAs take the SMs this grid's
-    // CTAs leave, and it waits for this grid before it exits.  (Behind the
+    // reads nothing this grid writes (with P.gs_merge, nothing before it has
+    // seen this grid's completion flag), so its CTAs take the SMs this
+    // grid's CTAs leave, and it waits for this grid before it exits.  (Behind the
     // generated-span pass instead, that pass has waited before it let this
     // grid launch; see the end of the kernel.)  No-ops for a plain launch.
     if (!P.prefix_after_gs) {
         asm volatile("griddepcontrol.wait;" ::: "memory");
+        // With merges in the generated-span pass, clear the completion flag
+        // that pass reads before it can launch (the last CTA of this grid
+        // to finish sets it; see the end of the kernel).
+        if (P.gs_merge) {
+            if (blockIdx.x == 0 && threadIdx.x == 0) {
+                atomicExch(P.sched + 4, 0u);
+                __threadfence();
+            }
+            __syncthreads();
+        }
         asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     }
     const uint32_t tmem = *s_tmem;
@@ -861,12 +872,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         asm volatile("griddepcontrol.wait;" ::: "memory");
     }
     // The last CTA to finish resets the work counter for the next launch
-    // (every CTA has claimed its last item before it gets here).
+    // (every CTA has claimed its last item before it gets here).  With
+    // merges in the generated-span pass it then sets the completion flag:
+    // every CTA fenced its partial states (written before the barrier above)
+    // before it counted itself, so a reader that sees the flag and then
+    // fences sees them all.
     if (threadIdx.x == 0) {
         __threadfence();
         if (atomicAdd(P.sched + 1, 1u) == gridDim.x - 1) {
             atomicExch(P.sched, 0u);
             atomicExch(P.sched + 1, 0u);
+            if (P.gs_merge) {
+                __threadfence();
+                atomicExch(P.sched + 4, 1u);
+            }
         }
     }
 }

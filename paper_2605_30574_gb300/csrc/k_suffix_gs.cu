@@ -68,6 +68,37 @@ __device__ __forceinline__ void bulk_copy(uint32_t dst, const void* src, uint32_
         : "memory");
 }
 
+__device__ __forceinline__ unsigned ld_relaxed_gpu(const unsigned* p) {
+    unsigned v;
+    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p));
+    return v;
+}
+
+// The merge of a row's two partial states -- the prompt-span pass's (when
+// has_span) and this pass's -- with a ZERO span's closed form, in exactly
+// the operations and order of the merge kernel for a row of at most two
+// states (merge_row.cuh): the same bits.  Returns the factor of the
+// weighted sum (0 for a row with nothing live) and the two weights.
+__device__ __forceinline__ float merge_two_weights(bool has_span, float2 ml_span, float m_gen, float l_gen,
+                                                   bool zero_span, int n_zero, float* w_span, float* w_gen) {
+    const bool live_s = has_span && ml_span.y > 0.f, live_g = l_gen > 0.f;
+    float M = fmaxf(live_s ? ml_span.x : -INFINITY, live_g ? m_gen : -INFINITY);
+    if (zero_span) M = fmaxf(M, 0.f);
+    *w_span = live_s ? exp2f(ml_span.x - M) : 0.f;
+    *w_gen = live_g ? exp2f(m_gen - M) : 0.f;
+    float den = __fadd_rn(has_span ? __fmul_rn(*w_span, ml_span.y) : 0.f, __fmul_rn(*w_gen, l_gen));
+    if (zero_span) den = fmaf(float(n_zero), exp2f(0.f - M), den);
+    return den > 0.f ? 1.f / den : 0.f;
+}
+
+__device__ __forceinline__ float merge_two(bool has_span, float w_span, float o_span, float w_gen, float o_gen,
+                                           float inv) {
+    float acc = 0.f;
+    if (has_span && w_span != 0.f) acc = fmaf(w_span, o_span, acc);
+    if (w_gen != 0.f) acc = fmaf(w_gen, o_gen, acc);
+    return __fmul_rn(acc, inv);
+}
+
 // The same without a cache hint: the query rows are read again by the
 // prompt-span pass of the call.
 __device__ __forceinline__ void bulk_copy_plain(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
@@ -167,8 +198,9 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
     // without a wait of its own, and it reads nothing this grid writes, so it
     // may take the SMs this grid's last CTAs leave.  (Behind the prompt-span
     // pass instead, that pass has waited before it let this grid launch, and
-    // this grid reads nothing it writes; see the end of the kernel.)  No-ops
-    // for a plain launch.
+    // this grid reads what it writes only after that pass's completion flag,
+    // with P.gs_merge; see the end of the kernel.)  No-ops for a plain
+    // launch.
     if (!P.gs_after_prefix) {
         asm volatile("griddepcontrol.wait;" ::: "memory");
         asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -300,12 +332,33 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
 
     int consumed = 0, cons_items = 0;
     bool ok = true;
+    bool ps_ready = false;   // the prompt-span pass's states are complete and visible
+    // This lane's dims after the key groups' reduce-scatter (below): F of
+    // the 16 it holds, from index `kept` on (round r keeps the upper half
+    // when bit r of gi is set); dims 8 c0 .. 8 c0 + 7 are the first 8 of
+    // the 16, 8 c1 .. 8 c1 + 7 the last 8.
+    constexpr int F = 16 / C::KPW;
+    // the merge path is built where its prompt-span states fit in registers
+    constexpr bool kCanMerge = GT * F <= 16;
+    int kept = 0;
+#pragma unroll
+    for (int r = 0; (C::LPK << r) < 32; ++r)
+        if ((gi >> r) & 1) kept += 8 >> r;
+    const int dim0 = kept < 8 ? 8 * c0 + kept : 8 * c1 + (kept - 8);
     for (int taken = 0; ok; ++taken) {
         __syncwarp();
         const int4 e0 = ring[2 * (taken & 3)];
         if (e0.x < 0) break;
         const int4 e1 = ring[2 * (taken & 3) + 1];
         const Item it{e0.x, e0.y, e0.z, e0.w, e1.x, e1.y, e1.z, e1.w};
+        // merges in this pass: the rows' source (a ZERO row needs no
+        // prompt-span state) and, until it has been seen set, the prompt-span
+        // pass's completion flag, read now and used at the item's end
+        unsigned code = 0, poll = 0;
+        if (kCanMerge && P.gs_merge) {
+            code = P.src[it.s];
+            if (!ps_ready) poll = ld_relaxed_gpu(P.sched + 4);
+        }
         // q rows of this item, pre-scaled into log2 units, as dim pairs: in
         // the item's query buffer once its first block has landed
         float2 q2[GT][8];
@@ -505,6 +558,43 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
         }
         if (!ok) break;
 
+        // ---- merge here?  Always for a ZERO row; for the others once the
+        // prompt-span pass has completed, whose states are fetched now (this
+        // lane's dims of every row), under the reduction below ----
+        bool merge_here = false;
+        const bool has_span = code != SPLICE_SRC_ZERO;
+        float2 ml_span[GT];
+        float o_span[GT][F];
+        if (kCanMerge && P.gs_merge) {
+            if (!ps_ready && __all_sync(kFull, poll != 0u)) {
+                asm volatile("fence.acq_rel.gpu;" ::: "memory");
+                ps_ready = true;
+            }
+            merge_here = !has_span || ps_ready;
+            if (merge_here && has_span) {
+#pragma unroll
+                for (int g = 0; g < GT; ++g) {
+                    const size_t row = size_t(it.s) * P.Hq + it.h * P.G + it.rc * GT + g;   // split 0's slot
+                    ml_span[g] = __ldcg(P.ws_ml + row);
+                    const float* sp = P.ws_o + row * D + dim0;
+                    if constexpr (F == 2) {
+                        const float2 t = __ldcg(reinterpret_cast<const float2*>(sp));
+                        o_span[g][0] = t.x;
+                        o_span[g][1] = t.y;
+                    } else {
+#pragma unroll
+                        for (int k = 0; k < F; k += 4) {
+                            const float4 t = __ldcg(reinterpret_cast<const float4*>(sp + k));
+                            o_span[g][k] = t.x;
+                            o_span[g][k + 1] = t.y;
+                            o_span[g][k + 2] = t.z;
+                            o_span[g][k + 3] = t.w;
+                        }
+                    }
+                }
+            }
+        }
+
         // ---- row sums of the group: the lanes holding distinct logits ----
         float l[GT];
 #pragma unroll
@@ -520,7 +610,6 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
         // max, and each keeps the half of its dims that its partner sends
         // it; after log2(KPW) rounds every lane holds F = 16 / KPW dims of
         // every row, summed over the groups, and m, l of every row ----
-        constexpr int F = 16 / C::KPW;
         float v[GT][16];
 #pragma unroll
         for (int g = 0; g < GT; ++g) {
@@ -530,7 +619,6 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
                 v[g][2 * i + 1] = o2[g][i].y;
             }
         }
-        int kept = 0;   // first of this lane's dims, as an index into its 16
 #pragma unroll
         for (int r = 0; (C::LPK << r) < 32; ++r) {
             const int off = C::LPK << r, W = 16 >> r;
@@ -552,12 +640,37 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
                 }
                 m[g] = M;
             }
-            if (hi) kept += W / 2;
         }
-        {
+        if (kCanMerge && merge_here) {
+            // the output, and the mark (l = -1 in this pass's slot) that
+            // tells the merge kernel the row is done
+            const bool zero_span = !has_span && P.p_hi > P.p_lo;
+#pragma unroll
+            for (int g = 0; g < GT; ++g) {
+                const size_t row = size_t(it.s) * P.Hq + it.h * P.G + it.rc * GT + g;
+                // the row's (m, l) as lane 0 would store it: the lanes' row
+                // sums can differ in the last bit (each lane adds its pair's
+                // two terms in its own order)
+                const float mg = __shfl_sync(kFull, m[g], 0), lg = __shfl_sync(kFull, l[g], 0);
+                float w_span, w_gen;
+                const float inv = merge_two_weights(has_span, has_span ? ml_span[g] : make_float2(-INFINITY, 0.f),
+                                                    mg, lg, zero_span, P.p_hi - P.p_lo, &w_span, &w_gen);
+                float r[F];
+#pragma unroll
+                for (int k = 0; k < F; ++k)
+                    r[k] = merge_two(has_span, w_span, has_span ? o_span[g][k] : 0.f, w_gen, v[g][k], inv);
+                float* op = P.out + row * D + dim0;
+                if constexpr (F == 2) {
+                    *reinterpret_cast<float2*>(op) = make_float2(r[0], r[1]);
+                } else {
+#pragma unroll
+                    for (int k = 0; k < F; k += 4)
+                        *reinterpret_cast<float4*>(op + k) = make_float4(r[k], r[k + 1], r[k + 2], r[k + 3]);
+                }
+                if (lane == 0) P.ws_ml[size_t(kMaxPrefixSplits) * P.B * P.Hq + row] = make_float2(0.f, -1.f);
+            }
+        } else {
             const int slot = kMaxPrefixSplits + it.split;
-            // dims 8 c0 .. 8 c0 + 7 are this lane's first 8, 8 c1 .. its last 8
-            const int dim0 = kept < 8 ? 8 * c0 + kept : 8 * c1 + (kept - 8);
 #pragma unroll
             for (int g = 0; g < GT; ++g) {
                 const size_t row = size_t(it.s) * P.Hq + it.h * P.G + it.rc * GT + g;
@@ -642,6 +755,11 @@ int generated_span_resident_warps(int d) {
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     // two 4-warp CTAs per SM (d <= 128), three 2-warp CTAs per SM (d = 256)
     return sms * (d == 256 ? 6 : 8);
+}
+
+bool generated_span_can_merge(int d, int G) {
+    const int gt = G % 4 == 0 ? 4 : (G % 2 == 0 ? 2 : 1);
+    return gt * d <= 512;   // GT * F <= 16 in gs_kernel, F = d / 32
 }
 
 int launch_generated_span(const AttnParams& p, void* stream, bool overlap_previous) {

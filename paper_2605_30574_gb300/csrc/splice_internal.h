@@ -112,8 +112,9 @@ struct AttnParams {
     const int32_t* dcount;        // [P][Dst][N][Hkv] encoded rows per span
     const int32_t* slot_delta;    // [num_slots] 1 = the slot is read in delta mode
     unsigned* err;
-    unsigned* sched;              // [4] prompt-span work counter and finished-CTA count, generated-span unit
-                                  // counter and finished-CTA count; zero between launches
+    unsigned* sched;              // [8]: [0], [1] prompt-span work counter and finished-CTA count, [2], [3]
+                                  // generated-span claim counter and finished-warp count (zero between
+                                  // launches); [4] prompt-span pass complete (gs_merge)
     int B, N, Hq, Hkv, D, G, Tp, T, Dst;
     int layer, step;
     int p_lo, p_hi, s_lo, s_hi;
@@ -123,6 +124,7 @@ struct AttnParams {
     int fuse_append;              // the generated-span pass also appends entry step - 1 (see kn, vn)
     int gs_after_prefix;          // the generated-span pass runs behind the prompt-span pass of the call
     int prefix_after_gs;          // the prompt-span pass runs behind the generated-span pass of the call
+    int gs_merge;                 // the generated-span pass merges rows itself (see launch_generated_span)
     int p_chunk, s_chunk;         // keys per split
     int n_tiles;
     int n_span_tiles;             // tiles [0, n_span_tiles) read stored spans, the rest delta rows
@@ -143,11 +145,15 @@ int launch_append(const uint16_t* kn, const uint16_t* vn, uint16_t* ks, uint16_t
 // work on the stream.  With p.gs_after_prefix = 0 the kernel is the call's
 // first and waits for that work before reading or writing anything, then
 // lets its dependents launch.  With 1 it directly follows the prompt-span
-// pass of the same call, which has already waited; it reads nothing that
-// pass writes, waits for it only before it exits, and lets its own
-// dependents launch only once its work is done.
+// pass of the same call, which has already waited; it reads what that pass
+// writes only with p.gs_merge, after it has seen that pass's completion
+// flag (sched[4]) and fenced, waits for it only before it exits, and lets
+// its own dependents launch only once its work is done.
 int launch_generated_span(const AttnParams& p, void* stream, bool overlap_previous);
 int generated_span_resident_warps(int d);
+// Whether the generated-span pass is built with its merge path for head
+// dim d and GQA group G (AttnParams::gs_merge may be set only then).
+bool generated_span_can_merge(int d, int G);
 // overlap_previous: the launch directly follows the last pass of the same
 // call on the stream (programmatic dependent launch; the kernel waits for it,
 // and that pass's completion implies the other pass's).

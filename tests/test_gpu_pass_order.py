@@ -1,10 +1,14 @@
 """The two attention passes in either order (and the order chosen per call)
 give the same outputs and the same generated-span store, bit for bit: the
-passes write disjoint partial states and the merge combines them in a fixed
-order (§3 attention over the prompt span and the generated span, Algorithm
-1's append).  Checked on a sweep where the prompt-span pass is small (the
-chosen order puts it first) and on the ladder-shaped sweep's full 512-sequence
-batch (the chosen order puts it second), with sampled rows against the oracle."""
+passes write disjoint partial states that are combined in a fixed order --
+by the merge kernel, or, with the prompt-span pass first and one split of
+each span, at the end of the generated-span items (ZERO rows always, the
+others once the prompt-span pass has completed), in the merge kernel's
+operations (§3 attention over the prompt span and the generated span,
+Algorithm 1's append).  Checked on a sweep where the prompt-span pass is
+small (the chosen order puts it first), on the ladder-shaped sweep's full
+512-sequence batch (the chosen order puts it second) and on head dims 64 and
+256, with sampled rows against the oracle."""
 import numpy as np
 import pytest
 import torch
@@ -75,6 +79,22 @@ def test_pass_order_ladder_batch():
     for s in (0, sb.B - 1):
         ref = oracle.decode_attn(wl, inp, s, sb.seqs[s], l, t)
         assert_close(out[s], ref, f"ladder s={s} l={l} t={t}")
+    sb.close()
+
+
+@pytest.mark.parametrize("name,points", [("tiny", [(0, 1), (2, 9), (3, 16)]),
+                                         ("gemma3-4b", [(0, 3), (5, 100), (33, 250)])])
+def test_pass_order_other_head_dims(name, points):
+    wl = WL.get(name)
+    sb = SweepBatch(wl, 0)
+    got = _run_orders(sb, points)
+    _check_equal(got, points)
+    inp = H.SynthInputs(wl)
+    l, t = points[-1]
+    out = got[1][-1][0].cpu().numpy()
+    for s in (0, sb.B // 2, sb.B - 1):
+        ref = oracle.decode_attn(wl, inp, s, sb.seqs[s], l, t)
+        assert_close(out[s], ref, f"{name} s={s} l={l} t={t}")
     sb.close()
 
 
