@@ -369,7 +369,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             int kj = 0, vj = 0;                  // block within the cursor's item
             ItemInfo ki{}, vi{};
             bool k_in = false, v_in = false, k_done = false, v_done = false;
+            // The next item is claimed when the K cursor issues the
+            // second-to-last block of its item (the claim's latency hides
+            // behind the last block's stage wait), so a CTA holds no item it
+            // will not start soon: claiming at the item's start left every
+            // CTA a whole item ahead, and near the end of the queue some CTAs
+            // still held two items while others had none.
             int nxt = int(atomicAdd(P.sched, 1u));
+            bool have_nxt = true;
             // a span's tiles read it at about the same time; afterwards its
             // lines go first, keeping the partial states in L2 for the merge
             const uint64_t pol = tc::l2_policy_evict_first();
@@ -381,6 +388,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (!k_in) {
                         const int r = kpost % kItemRing;
                         if (tc::mbar_test_wait(bar(Bb::IEMPTY + r), (uint32_t(kpost / kItemRing) & 1u) ^ 1u)) {
+                            if (!have_nxt) nxt = int(atomicAdd(P.sched, 1u));   // an item with no block
+                            have_nxt = false;
                             const int item = nxt < tp.n_items ? nxt : -1;
                             ItemInfo inf;
                             inf.item = -1;
@@ -392,7 +401,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                             if (item < 0) {
                                 k_done = true;
                             } else {
-                                nxt = int(atomicAdd(P.sched, 1u));   // claimed now, needed at the next item
                                 ki = inf;
                                 kj = 0;
                                 k_in = true;
@@ -413,6 +421,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                             ++kg;
                             ++kj;
                             prog = true;
+                            if (!have_nxt && kj >= ki.nblk - 1) {
+                                nxt = int(atomicAdd(P.sched, 1u));
+                                have_nxt = true;
+                            }
                         }
                     }
                 }
