@@ -320,12 +320,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     // grid launch; see the end of the kernel.)  No-ops for a plain launch.
     if (!P.prefix_after_gs) {
         asm volatile("griddepcontrol.wait;" ::: "memory");
-        // With merges in the generated-span pass, clear the completion flag
-        // that pass reads before it can launch (the last CTA of this grid
-        // to finish sets it; see the end of the kernel).
-        if (P.gs_merge) {
+        // The generated-span pass queued behind this grid claims its items
+        // from a counter (sched[2]) and, with merges, reads this grid's
+        // completion flag (sched[4]; the last CTA to finish sets it, see the
+        // end of the kernel): both are cleared before that pass can launch.
+        if (P.gs_after_prefix) {
             if (blockIdx.x == 0 && threadIdx.x == 0) {
-                atomicExch(P.sched + 4, 0u);
+                atomicExch(P.sched + 2, 0u);
+                if (P.gs_merge) atomicExch(P.sched + 4, 0u);
                 __threadfence();
             }
             __syncthreads();

@@ -232,7 +232,8 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
     // start as that pass's CTAs leave) every later item is claimed from the
     // launch-wide counter (numbered from the grid's warp count on), one
     // ahead: lane 0 holds the claim in flight, whose value is needed only
-    // when the next item starts ----
+    // when the next item starts (the prompt-span pass clears the counter
+    // before this grid can launch) ----
     const unsigned nwarps = gridDim.x * C::WARPS;
     // The warps' ranks.  With the prompt-span pass queued behind, SM-major
     // when the grid is whole waves of sm_count CTAs: the first wave's CTAs
@@ -707,17 +708,8 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
         asm volatile("griddepcontrol.wait;" ::: "memory");
         asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     }
-    // Run-time claims: the last warp to finish resets the item counter for
-    // the next launch (every warp's claims have all returned before it gets
-    // here: the one in flight when its last item started came back past the
-    // end and ended its walk).
-    if (claims && lane == 0) {
-        __threadfence();
-        if (atomicAdd(P.sched + 3, 1u) == nwarps - 1) {
-            atomicExch(P.sched + 2, 0u);
-            atomicExch(P.sched + 3, 0u);
-        }
-    }
+    // (Run-time claims: the prompt-span pass ahead of this grid cleared the
+    // item counter before this grid could launch.)
 }
 
 template <int D, int GT>

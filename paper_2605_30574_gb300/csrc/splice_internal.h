@@ -112,9 +112,9 @@ struct AttnParams {
     const int32_t* dcount;        // [P][Dst][N][Hkv] encoded rows per span
     const int32_t* slot_delta;    // [num_slots] 1 = the slot is read in delta mode
     unsigned* err;
-    unsigned* sched;              // [8]: [0], [1] prompt-span work counter and finished-CTA count, [2], [3]
-                                  // generated-span claim counter and finished-warp count (zero between
-                                  // launches); [4] prompt-span pass complete (gs_merge)
+    unsigned* sched;              // [8]: [0], [1] prompt-span work counter and finished-CTA count (zero
+                                  // between launches); [2] generated-span claim counter and [4] prompt-span
+                                  // pass complete (gs_merge), both cleared by the prompt-span pass ahead
     int B, N, Hq, Hkv, D, G, Tp, T, Dst;
     int layer, step;
     int p_lo, p_hi, s_lo, s_hi;
