@@ -886,13 +886,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         asm volatile("griddepcontrol.wait;" ::: "memory");
     }
     // The last CTA to finish resets the work counter for the next launch
-    // (every CTA has claimed its last item before it gets here).  With
-    // merges in the generated-span pass it then sets the completion flag:
-    // every CTA fenced its partial states (written before the barrier above)
-    // before it counted itself, so a reader that sees the flag and then
-    // fences sees them all.
+    // (every CTA's claims have returned before it gets here, so they are
+    // performed).  With merges in the generated-span pass it then sets the
+    // completion flag: every CTA fenced its partial states (written before
+    // the barrier above) before it counted itself, so a reader that sees
+    // the flag and then fences sees them all.
     if (threadIdx.x == 0) {
-        __threadfence();
+        if (P.gs_merge) __threadfence();
         if (atomicAdd(P.sched + 1, 1u) == gridDim.x - 1) {
             atomicExch(P.sched, 0u);
             atomicExch(P.sched + 1, 0u);

@@ -113,8 +113,9 @@ struct AttnParams {
     const int32_t* slot_delta;    // [num_slots] 1 = the slot is read in delta mode
     unsigned* err;
     unsigned* sched;              // [8]: [0], [1] prompt-span work counter and finished-CTA count (zero
-                                  // between launches); [2] generated-span claim counter and [4] prompt-span
-                                  // pass complete (gs_merge), both cleared by the prompt-span pass ahead
+                                  // between launches); [2] generated-span claim counter and [4]
+                                  // prompt-span pass complete (gs_merge), both cleared by the prompt-span
+                                  // pass ahead
     int B, N, Hq, Hkv, D, G, Tp, T, Dst;
     int layer, step;
     int p_lo, p_hi, s_lo, s_hi;
