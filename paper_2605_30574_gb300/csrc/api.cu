@@ -474,10 +474,10 @@ splice_status attn_common(splice_desc* d, int layer, int step, const splice_bf16
     p.prefix_after_gs = gs_work && prefix_launched && !prefix_first && !d->profiling ? 1 : 0;
     // Behind the prompt-span pass, with one prompt-span and one
     // generated-span split per row and no delta rows, the generated-span
-    // pass merges each item's rows itself -- ZERO rows always, the others
-    // once the prompt-span pass has completed (a flag it reads without
-    // waiting) -- writes the output and marks the row; the merge kernel
-    // then only merges the rows left unmarked.
+    // pass merges every row itself and writes the output: ZERO rows at the
+    // item's end, the others there once the prompt-span pass has completed
+    // (a flag it reads without waiting), else at the warp's end after the
+    // grid dependency wait.  No merge kernel is launched then.
     p.gs_merge = p.gs_after_prefix && p.nss == 1 && p.nsp == 1 && !p.delta_on &&
                          splice::generated_span_can_merge(sh.head_dim, p.G)
                      ? 1
@@ -523,6 +523,7 @@ splice_status attn_common(splice_desc* d, int layer, int step, const splice_bf16
         const splice_status st = launch_prefix();
         if (st != SPLICE_OK) return st;
     }
+    if (p.gs_merge) return SPLICE_OK;
     const bool merge_overlap = (prefix_launched || gs_work) && !d->profiling;
     e = timed_launch(d, 3, stream, [&] { return splice::launch_merge(p, stream, merge_overlap); });
     if (e != cudaSuccess) return cuda_fail(e, "merge launch");

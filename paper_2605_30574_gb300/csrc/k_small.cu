@@ -48,13 +48,11 @@ __global__ void __launch_bounds__(256, 5) merge_kernel(AttnParams P) {
     if constexpr (D <= 128) {
         const long row0 = 2 * warp;
         if (row0 >= total) return;
-        const unsigned skip = merged_rows<2>(P, row0, lane);
-        if (merge_rows_fast2<D, 4>(P, row0, lane, skip)) return;
-        if (!(skip & 1u)) merge_row(P, row0, lane);
-        if (row0 + 1 < total && !(skip & 2u)) merge_row(P, row0 + 1, lane);
+        if (merge_rows_fast2<D, 4>(P, row0, lane)) return;
+        merge_row(P, row0, lane);
+        if (row0 + 1 < total) merge_row(P, row0 + 1, lane);
     } else {
         if (warp >= total) return;
-        if (merged_rows<1>(P, warp, lane)) return;
         if (!merge_row_fast<D, 4>(P, warp, lane)) merge_row(P, warp, lane);
     }
 }
@@ -71,17 +69,12 @@ __global__ void __launch_bounds__(256, 3) merge_kernel4(AttnParams P) {
     const long total = long(P.B) * P.Hq;
     const long row0 = 4 * warp;
     if (row0 >= total) return;
-    const unsigned skip = merged_rows<4>(P, row0, lane);
-    const unsigned live = total - row0 >= 4 ? 0xfu : (1u << (total - row0)) - 1u;
-    if ((skip & live) == live) return;
-    if (merge_rows_group<D, 2, 4>(P, row0, lane, skip)) return;
-    for (long r = row0; r < row0 + 4 && r < total; r += 2) {
-        const unsigned sk = (skip >> (r - row0)) & 3u;
-        if (!merge_rows_fast2<D, 4>(P, r, lane, sk)) {
-            if (!(sk & 1u)) merge_row(P, r, lane);
-            if (r + 1 < total && !(sk & 2u)) merge_row(P, r + 1, lane);
+    if (merge_rows_group<D, 2, 4>(P, row0, lane)) return;
+    for (long r = row0; r < row0 + 4 && r < total; r += 2)
+        if (!merge_rows_fast2<D, 4>(P, r, lane)) {
+            merge_row(P, r, lane);
+            if (r + 1 < total) merge_row(P, r + 1, lane);
         }
-    }
 }
 
 }  // namespace

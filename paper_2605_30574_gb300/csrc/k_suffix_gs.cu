@@ -107,6 +107,10 @@ __device__ __forceinline__ void bulk_copy_plain(uint32_t dst, const void* src, u
                  : "memory");
 }
 
+// Items a warp may leave unmerged until its end (with P.gs_merge): those
+// that end before the prompt-span pass has completed.
+constexpr int kPend = 8;
+
 template <int D, int GT>
 struct GS {
     static constexpr int LPK = D / 16;              // lanes per key
@@ -130,7 +134,8 @@ struct GS {
     static constexpr uint32_t OFF_TAKEN = OFF_BAR + 16;       // [4] items (decoded) in the order the issue cursor took them
     static constexpr uint32_t QROWS = GT * D * 2;             // the GT query rows of one item
     static constexpr uint32_t OFF_Q = OFF_TAKEN + 4 * 32;     // [2] query rows, brought with each item's first block
-    static constexpr uint32_t PER_WARP = (OFF_Q + 2 * QROWS + 127) / 128 * 128;
+    static constexpr uint32_t OFF_PEND = OFF_Q + 2 * QROWS;   // [kPend] items whose merge waits for the warp's end
+    static constexpr uint32_t PER_WARP = (OFF_PEND + kPend * 4 + 127) / 128 * 128;
     static constexpr uint32_t SMEM = WARPS * PER_WARP;
     static_assert(NV % 4 == 0 || NV < 4, "reduce layout");
     static_assert(NV < LPK || NV == VPL * LPK, "every logit of a group owned by one lane");
@@ -211,6 +216,8 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
     float* red = reinterpret_cast<float*>(ws + C::OFF_RED);
     float2* pp = reinterpret_cast<float2*>(ws + C::OFF_PP);
     int4* ring = reinterpret_cast<int4*>(ws + C::OFF_TAKEN);
+    int* pend = reinterpret_cast<int*>(ws + C::OFF_PEND);
+    int npend = 0;
 
     const int gi = lane / C::LPK, dl = lane % C::LPK;
     const int g_mine = dl % GT;
@@ -587,7 +594,10 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
 
         // ---- merge here?  Always for a ZERO row; for the others once the
         // prompt-span pass has completed, whose states are fetched now (this
-        // lane's dims of every row), under the reduction below ----
+        // lane's dims of every row), under the reduction below.  An item
+        // that ends before then writes its partial state and is merged at
+        // the warp's end (up to kPend of them; past that the warp waits
+        // for the prompt-span grid here) ----
         bool merge_here = false;
         const bool has_span = code != SPLICE_SRC_ZERO;
         float2 ml_span[GT];
@@ -598,6 +608,16 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
                 ps_ready = true;
             }
             merge_here = !has_span || ps_ready;
+            if (!merge_here) {
+                if (npend < kPend) {
+                    if (lane == 0) pend[npend] = it.idx;
+                    ++npend;
+                } else {
+                    asm volatile("griddepcontrol.wait;" ::: "memory");
+                    ps_ready = true;
+                    merge_here = true;
+                }
+            }
             if (merge_here && has_span) {
 #pragma unroll
                 for (int g = 0; g < GT; ++g) {
@@ -669,8 +689,7 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
             }
         }
         if (kCanMerge && merge_here) {
-            // the output, and the mark (l = -1 in this pass's slot) that
-            // tells the merge kernel the row is done
+            // the output
             const bool zero_span = !has_span && P.p_hi > P.p_lo;
 #pragma unroll
             for (int g = 0; g < GT; ++g) {
@@ -694,7 +713,6 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
                     for (int k = 0; k < F; k += 4)
                         *reinterpret_cast<float4*>(op + k) = make_float4(r[k], r[k + 1], r[k + 2], r[k + 3]);
                 }
-                if (lane == 0) P.ws_ml[size_t(kMaxPrefixSplits) * P.B * P.Hq + row] = make_float2(0.f, -1.f);
             }
         } else {
             const int slot = kMaxPrefixSplits + it.split;
@@ -726,12 +744,49 @@ __global__ void __launch_bounds__(GS<D, GT>::WARPS * 32)
     }
     if (P.gs_after_prefix) {
         // Behind the prompt-span pass: this grid's completion must imply that
-        // pass's, so the merge queued behind this grid sees both.  Then the
-        // merge may launch (it waits for this whole grid before it reads
-        // anything); every CTA of this grid is running by the time all of
-        // them have signalled, so the merge's CTAs never hold an SM it still
-        // needs.
+        // pass's, so the merge queued behind this grid sees both (with
+        // P.gs_merge no merge is queued: this grid writes every output).
+        // Then the work behind may launch (the merge waits for this whole
+        // grid before it reads anything); every CTA of this grid is running
+        // by the time all of them have signalled, so those CTAs never hold
+        // an SM it still needs.
         asm volatile("griddepcontrol.wait;" ::: "memory");
+        // The items left unmerged: the prompt-span states are complete and
+        // visible now; this warp's own partial states are re-read (the same
+        // bits it stored) and merged as at an item's end.
+        if constexpr (kCanMerge) {
+            if (P.gs_merge && npend > 0) {
+                __syncwarp();
+                for (int k = 0; k < npend; ++k) {
+                    Item it;
+                    item_of(P, dv, pend[k], it);
+#pragma unroll
+                    for (int g = 0; g < GT; ++g) {
+                        const size_t row = size_t(it.s) * P.Hq + it.h * P.G + it.rc * GT + g;
+                        const size_t gen = size_t(kMaxPrefixSplits) * P.B * P.Hq + row;
+                        const float2 ml_gen = __ldcg(P.ws_ml + gen), ml_span = __ldcg(P.ws_ml + row);
+                        float og[F], os[F];
+#pragma unroll
+                        for (int j = 0; j < F; j += 2) {
+                            const float2 a = __ldcg(reinterpret_cast<const float2*>(P.ws_o + gen * D + dim0 + j));
+                            const float2 b = __ldcg(reinterpret_cast<const float2*>(P.ws_o + row * D + dim0 + j));
+                            og[j] = a.x;
+                            og[j + 1] = a.y;
+                            os[j] = b.x;
+                            os[j + 1] = b.y;
+                        }
+                        float w_span, w_gen;
+                        const float inv = merge_two_weights(true, ml_span, ml_gen.x, ml_gen.y, false, 0, &w_span, &w_gen);
+                        float* op = P.out + row * D + dim0;
+#pragma unroll
+                        for (int j = 0; j < F; j += 2)
+                            *reinterpret_cast<float2*>(op + j) = make_float2(merge_two(true, w_span, os[j], w_gen, og[j], inv),
+                                                                             merge_two(true, w_span, os[j + 1], w_gen,
+                                                                                       og[j + 1], inv));
+                    }
+                }
+            }
+        }
         asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     }
     // (Run-time claims: the prompt-span pass ahead of this grid cleared the

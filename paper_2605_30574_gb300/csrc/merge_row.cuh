@@ -114,10 +114,9 @@ __device__ __forceinline__ bool merge_row_fast(const AttnParams& P, long row, in
 // the row's lanes with the partials on its first n lanes, so they add the
 // same values in the same order as merge_weights over 32 lanes (the other
 // lanes hold zeros): the same bits as merge_row_fast.  False (nothing
-// written) if any of the rows has more partials.  Bit r of `skip`: row
-// row0 + r is done already (neither read nor written).
+// written) if any of the rows has more partials.
 template <int D, int NF, int RPW>
-__device__ __forceinline__ bool merge_rows_group(const AttnParams& P, long row0, int lane, unsigned skip = 0u) {
+__device__ __forceinline__ bool merge_rows_group(const AttnParams& P, long row0, int lane) {
     constexpr int LPR = 32 / RPW;                // lanes per row
     static_assert(NF <= LPR, "a row's partials sit on its first lanes");
     constexpr int C4 = D / 4;                    // float4 slices of a row
@@ -125,7 +124,7 @@ __device__ __forceinline__ bool merge_rows_group(const AttnParams& P, long row0,
     const int half = lane / LPR, hl = lane % LPR;
     const long total = long(P.B) * P.Hq;
     const long row = row0 + half;
-    const bool live_row = row < total && !((skip >> half) & 1u);
+    const bool live_row = row < total;
     RowParts rp{0, 0, 0};
     uint8_t code = SPLICE_SRC_CLEAN;
     if (live_row) {
@@ -187,20 +186,8 @@ __device__ __forceinline__ bool merge_rows_group(const AttnParams& P, long row0,
 }
 
 template <int D, int NF>
-__device__ __forceinline__ bool merge_rows_fast2(const AttnParams& P, long row0, int lane, unsigned skip = 0u) {
-    return merge_rows_group<D, NF, 2>(P, row0, lane, skip);
-}
-
-// Rows the generated-span pass merged itself (P.gs_merge) carry l = -1 in
-// its partial slot: bit i of the result is set when row row0 + i (i < RPW)
-// is such a row.  Every lane of the warp must call it.
-template <int RPW>
-__device__ __forceinline__ unsigned merged_rows(const AttnParams& P, long row0, int lane) {
-    if (!P.gs_merge) return 0u;
-    const long total = long(P.B) * P.Hq;
-    const long r = row0 + lane % RPW;
-    const bool done = r < total && __ldcg(P.ws_ml + size_t(kMaxPrefixSplits) * total + r).y < 0.f;
-    return __ballot_sync(0xffffffffu, done) & ((1u << RPW) - 1u);
+__device__ __forceinline__ bool merge_rows_fast2(const AttnParams& P, long row0, int lane) {
+    return merge_rows_group<D, NF, 2>(P, row0, lane);
 }
 
 // Any number of live partials (up to kMaxSplits): weights first, then the o
