@@ -360,8 +360,9 @@ splice_status splice_plan_stats(const splice_desc* desc, int layer, int step, in
  * 2 the generated-span pass first.  Outputs and stores are bit-identical in
  * every order (the passes write disjoint partial states that are combined
  * in a fixed order, by the merge kernel or -- with the prompt-span pass
- * first -- at the end of a generated-span item once the prompt-span pass
- * has completed); only the overlap of the two passes changes.
+ * first and one split of each span -- by the generated-span pass once the
+ * prompt-span pass has completed); only the overlap of the two passes
+ * changes.
  * SPLICE_EINVAL for another value.  No device work.
  */
 splice_status splice_debug_pass_order(splice_desc* desc, int order);

@@ -2,9 +2,9 @@
 give the same outputs and the same generated-span store, bit for bit: the
 passes write disjoint partial states that are combined in a fixed order --
 by the merge kernel, or, with the prompt-span pass first and one split of
-each span, at the end of the generated-span items (ZERO rows always, the
-others once the prompt-span pass has completed), in the merge kernel's
-operations (§3 attention over the prompt span and the generated span,
+each span, by the generated-span pass (ZERO rows at an item's end, the
+others there once the prompt-span pass has completed, else at the warp's
+end), in the merge kernel's operations (§3 attention over the prompt span and the generated span,
 Algorithm 1's append).  Checked on a sweep where the prompt-span pass is
 small (the chosen order puts it first), on the ladder-shaped sweep's full
 512-sequence batch (the chosen order puts it second) and on head dims 64 and
