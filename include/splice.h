@@ -356,7 +356,8 @@ splice_status splice_plan_stats(const splice_desc* desc, int layer, int step, in
  * splice_debug_pass_order -- order of the two attention passes in later
  * calls on the descriptor: 0 (the default) chosen per call from the plan --
  * the prompt-span pass first when it holds fewer than 3072 keys per SM
- * (summed over its items), else the generated-span pass first; 1 the prompt-span pass first;
+ * (summed over its items) or more than twice the generated-span pass's
+ * keys, else the generated-span pass first; 1 the prompt-span pass first;
  * 2 the generated-span pass first.  Outputs and stores are bit-identical in
  * every order (the passes write disjoint partial states that are combined
  * in a fixed order, by the merge kernel or -- with the prompt-span pass

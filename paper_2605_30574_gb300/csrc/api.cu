@@ -456,8 +456,11 @@ splice_status attn_common(splice_desc* d, int layer, int step, const splice_bf16
     // fill the generated-span pass's tail.  A smaller prompt-span pass goes
     // first: its short run and its tail (part of the SMs idle while its last
     // items finish) are filled by the generated-span pass's run-time claimed
-    // items.  With per-launch timing on, the events between the launches
-    // serialise everything.
+    // items.  So does a prompt-span pass with more than
+    // kPrefixFirstGenRatio times the generated-span pass's keys (x row
+    // chunks): the generated-span pass's short items then fill its tail.
+    // With per-launch timing on, the events between the launches serialise
+    // everything.
     const bool gs_work = p.nss > 0;
     const long prefix_items = long(p.n_span_tiles) * sh.num_kv_heads * p.nsp +
                               long(p.n_tiles - p.n_span_tiles) * sh.num_kv_heads * p.nsd;
@@ -467,9 +470,12 @@ splice_status attn_common(splice_desc* d, int layer, int step, const splice_bf16
         (long(p.n_span_tiles) * ((p_vis + box - 1) / box) +
          long(p.n_tiles - p.n_span_tiles) * (p.nsd ? (d->delta_max + box - 1) / box : 0)) *
         sh.num_kv_heads * box;
+    const long gs_keys = long(d->B) * sh.num_kv_heads * (p.G / (p.G % 4 == 0 ? 4 : (p.G % 2 == 0 ? 2 : 1))) * s_vis;
     const bool prefix_first =
-        prefix_launched && (d->pass_order == 1 ||
-                            (d->pass_order == 0 && prefix_keys < long(d->sms) * splice::kPrefixFirstKeysPerSm));
+        prefix_launched &&
+        (d->pass_order == 1 ||
+         (d->pass_order == 0 && (prefix_keys < long(d->sms) * splice::kPrefixFirstKeysPerSm ||
+                                 gs_keys * splice::kPrefixFirstGenRatio < prefix_keys)));
     p.gs_after_prefix = gs_work && prefix_launched && prefix_first && !d->profiling ? 1 : 0;
     p.prefix_after_gs = gs_work && prefix_launched && !prefix_first && !d->profiling ? 1 : 0;
     // Behind the prompt-span pass, with one prompt-span and one

@@ -27,6 +27,9 @@ constexpr int kPrefixSplitKeys = 1024;
 // The call's prompt-span pass goes first when it holds fewer than this many
 // keys (summed over its items) per SM.
 constexpr int kPrefixFirstKeysPerSm = 3072;
+// It also goes first when its keys exceed kPrefixFirstGenRatio x the
+// generated-span pass's (keys x row chunks).
+constexpr int kPrefixFirstGenRatio = 2;
 // Group source flag: the group reads the delta-encoded rows of a donor slot
 // (group_src = kGroupDelta | (SPLICE_SRC_DONOR0 + slot)).
 constexpr int32_t kGroupDelta = SPLICE_GROUP_DELTA;

@@ -7,8 +7,8 @@ others there once the prompt-span pass has completed, else at the warp's
 end), in the merge kernel's operations (§3 attention over the prompt span and the generated span,
 Algorithm 1's append).  Checked on a sweep where the prompt-span pass is
 small (the chosen order puts it first), on the ladder-shaped sweep's full
-512-sequence batch (the chosen order puts it second) and on head dims 64 and
-256, with sampled rows against the oracle."""
+512-sequence batch (at t = 700 the chosen order puts it second) and on head
+dims 64 and 256, with sampled rows against the oracle."""
 import numpy as np
 import pytest
 import torch
