@@ -102,13 +102,6 @@ __device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&v)[8])
                  : "memory");
 }
 
-// 8 floats to global memory in one 256-bit store (32-byte aligned address).
-__device__ __forceinline__ void st_global_v8(float* p, const float* v) {
-    asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "f"(v[0]), "f"(v[1]),
-                 "f"(v[2]), "f"(v[3]), "f"(v[4]), "f"(v[5]), "f"(v[6]), "f"(v[7])
-                 : "memory");
-}
-
 // One segment's P (bf16 pairs), by segment size.
 __device__ __forceinline__ void store_p(uint32_t taddr, const uint32_t (&v)[16]) { tmem_st16(taddr, v); }
 __device__ __forceinline__ void store_p(uint32_t taddr, const uint32_t (&v)[8]) { tmem_st8(taddr, v); }
@@ -143,7 +136,11 @@ struct Cfg {
     static constexpr uint32_t X_BYTES = 2 * (2 * 2 * kRows) * 4;
     static constexpr uint32_t OFF_BAR = OFF_X + X_BYTES;
     static constexpr uint32_t OFF_RING = OFF_BAR + 1024;    // [kItemRing] posted work items
-    static constexpr uint32_t SMEM = OFF_RING + kItemRing * kRingEntryBytes + 1024;   // + alignment slack
+    // [8 softmax warps][32 rows][16 floats]: the epilogue's staging, so the
+    // partial states leave in row-contiguous 64-byte pieces
+    static constexpr uint32_t OFF_STG = (OFF_RING + kItemRing * kRingEntryBytes + 127) / 128 * 128;
+    static constexpr uint32_t STG_BYTES = 32 * 16 * 4;
+    static constexpr uint32_t SMEM = OFF_STG + 8 * STG_BYTES + 1024;   // + alignment slack
     static_assert(NSLOT >= 2 && COL_O + D <= kTmemCols, "TMEM budget");
     static_assert(SMEM <= 227 * 1024, "shared memory budget");
     static_assert(KPT % 32 == 0 && OCH % 32 == 0 && VST >= 2, "TMEM access granularity, ring depth");
@@ -836,15 +833,45 @@ __global__ void __launch_bounds__(kThreads, 1)
             float* xb = xl + (k & 1) * (2 * kRows);
             if (it.nblk > 0) {
                 if (rows) {
-                    float* op = P.ws_o + idx * D + wg * C::OCH;
+                    // Each thread holds its row's half of O.  Stores of one
+                    // value per thread would touch 32 rows (lines) per
+                    // instruction, so the warp stages 16 columns of its 32
+                    // rows at a time in shared memory and stores them as 8
+                    // rows x 64 contiguous bytes per instruction (16-byte
+                    // units rotated by row pair, so neither side conflicts).
+                    // (a partial-state index fits in 32 bits: the workspace holds 16 x
+                    // rows x 520 bytes, far below 2^31 rows of device memory)
+                    const int my_idx = valid ? int(idx) : -1;
+                    int ridx[4];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) ridx[i] = __shfl_sync(0xffffffffu, my_idx, i * 8 + lane / 4);
+                    float* stg = reinterpret_cast<float*>(smem + C::OFF_STG + (warp - 4) * C::STG_BYTES);
+                    const int u = lane & 3;
 #pragma unroll
                     for (int q = 0; q < C::OCH / 32; ++q) {
                         float v[32];
                         tc::tmem_ld32(tmem + lane_base + C::COL_O + wg * C::OCH + q * 32, v);
                         tc::tmem_wait_ld();
-                        if (valid) {
 #pragma unroll
-                            for (int i = 0; i < 32; i += 8) st_global_v8(op + q * 32 + i, v + i);
+                        for (int h = 0; h < 2; ++h) {
+#pragma unroll
+                            for (int w = 0; w < 4; ++w) {
+                                const int slot = (w + (lane >> 1)) & 3;
+                                *reinterpret_cast<float4*>(stg + lane * 16 + slot * 4) =
+                                    make_float4(v[h * 16 + w * 4], v[h * 16 + w * 4 + 1], v[h * 16 + w * 4 + 2],
+                                                v[h * 16 + w * 4 + 3]);
+                            }
+                            __syncwarp();
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                const int r = i * 8 + lane / 4;
+                                const float4 x =
+                                    *reinterpret_cast<const float4*>(stg + r * 16 + ((u + (r >> 1)) & 3) * 4);
+                                if (ridx[i] >= 0)
+                                    *reinterpret_cast<float4*>(P.ws_o + size_t(ridx[i]) * D + wg * C::OCH + q * 32 +
+                                                               h * 16 + u * 4) = x;
+                            }
+                            __syncwarp();
                         }
                     }
                 }
