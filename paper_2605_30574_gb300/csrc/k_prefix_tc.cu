@@ -651,9 +651,92 @@ __global__ void __launch_bounds__(kThreads, 1)
         constexpr int SEG = KPT / 2;                   // keys per row-sum segment
         const int row = quarter * 32 + lane;           // == TMEM lane of this thread's row
         int jg = 0;
+        // An item's epilogue (its partial states out of O, then O freed).
+        // For d = 256 (64-key blocks, half as long) it is deferred past the
+        // next item's first block, whose softmax then runs while the item's
+        // last P V completes (a Gemma-3-4B-shaped sweep +1.4%); for d <= 128
+        // that held O, and so the next item's first P V, too long for the
+        // three S slots to cover (the ladder -1.3%).  The item's state:
+        constexpr bool kDefer = D == 256;
+        bool pend = false, pend_full = false, pend_rows = false;
+        int pend_k = 0, pend_idx = -1;                 // pend_idx: -1 for a row outside the tile
+        float pend_m = 0.f, pend_l = 0.f;
+        auto epilogue = [&]() -> bool {
+            pend = false;
+            // Every thread waits for the item's O before it frees it, so
+            // arrivals of one item never land in an earlier item's phase.
+            if (!__all_sync(0xffffffffu,
+                            tc::mbar_wait(bar(Bb::ODONE), uint32_t(pend_k) & 1u, s_abort, P.err, kErrWaitSoftmax)))
+                return false;
+            tc::tc_fence_after();
+            float* xb = xl + (pend_k & 1) * (2 * kRows);
+            if (pend_full) {
+                if (pend_rows) {
+                    // Each thread holds its row's half of O.  Stores of one
+                    // value per thread would touch 32 rows (lines) per
+                    // instruction, so the warp stages 16 columns of its 32
+                    // rows at a time in shared memory and stores them as 8
+                    // rows x 64 contiguous bytes per instruction (16-byte
+                    // units rotated by row pair, so neither side conflicts).
+                    int ridx[4];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) ridx[i] = __shfl_sync(0xffffffffu, pend_idx, i * 8 + lane / 4);
+                    float* stg = reinterpret_cast<float*>(smem + C::OFF_STG + (warp - 4) * C::STG_BYTES);
+                    const int u = lane & 3;
+#pragma unroll
+                    for (int q = 0; q < C::OCH / 32; ++q) {
+                        float v[32];
+                        tc::tmem_ld32(tmem + lane_base + C::COL_O + wg * C::OCH + q * 32, v);
+                        tc::tmem_wait_ld();
+#pragma unroll
+                        for (int h = 0; h < 2; ++h) {
+#pragma unroll
+                            for (int w = 0; w < 4; ++w) {
+                                const int slot = (w + (lane >> 1)) & 3;
+                                *reinterpret_cast<float4*>(stg + lane * 16 + slot * 4) =
+                                    make_float4(v[h * 16 + w * 4], v[h * 16 + w * 4 + 1], v[h * 16 + w * 4 + 2],
+                                                v[h * 16 + w * 4 + 3]);
+                            }
+                            __syncwarp();
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                const int r = i * 8 + lane / 4;
+                                const float4 x =
+                                    *reinterpret_cast<const float4*>(stg + r * 16 + ((u + (r >> 1)) & 3) * 4);
+                                if (ridx[i] >= 0)
+                                    *reinterpret_cast<float4*>(P.ws_o + size_t(ridx[i]) * D + wg * C::OCH + q * 32 +
+                                                               h * 16 + u * 4) = x;
+                            }
+                            __syncwarp();
+                        }
+                    }
+                }
+                xb[wg * kRows + row] = pend_l;
+                tc::mbar_arrive(bar(Bb::LXCH));
+                if (!__all_sync(0xffffffffu,
+                                tc::mbar_wait(bar(Bb::LXCH), uint32_t(pend_k) & 1u, s_abort, P.err, kErrWaitSoftmax)))
+                    return false;
+                if (wg == 0 && pend_idx >= 0) P.ws_ml[pend_idx] = make_float2(pend_m, xb[row] + xb[kRows + row]);
+            } else {
+                // an empty split: a state with no keys (still one exchange
+                // round, so every item moves the exchange barrier once)
+                tc::mbar_arrive(bar(Bb::LXCH));
+                if (!__all_sync(0xffffffffu,
+                                tc::mbar_wait(bar(Bb::LXCH), uint32_t(pend_k) & 1u, s_abort, P.err, kErrWaitSoftmax)))
+                    return false;
+                if (wg == 0 && pend_idx >= 0) P.ws_ml[pend_idx] = make_float2(-INFINITY, 0.f);
+            }
+            tc::tc_fence_before();
+            tc::mbar_arrive(bar(Bb::OFREE));
+            return true;
+        };
+        bool ok = true;
         for (int k = 0;; ++k) {
             const ItemInfo it = take_item(k);
-            if (it.item < 0) break;
+            if (it.item < 0) {
+                ok = it.item == -1;
+                break;
+            }
             const int nrows = it.nseq * P.G;
             const bool rows = quarter * 32 < nrows;    // warp-uniform
             const bool valid = row < nrows;
@@ -671,7 +754,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             // row sum kept per segment of this thread's keys (two), added at
             // the item's end
             float m_run = -INFINITY, l_seg0 = 0.f, l_seg1 = 0.f;
-            bool ok = true;
             for (int j = 0; j < it.nblk; ++j, ++jg) {
                 const int slot = jg % NSLOT;
                 // waits are made warp-uniform: tcgen05.ld/st are warp-collective
@@ -819,82 +901,39 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 tc::tc_fence_before();
                 tc::mbar_arrive(bar(Bb::PFULL + slot));
+                // the previous item's epilogue, now that this item's first P
+                // is out
+                if (kDefer && pend && !epilogue()) {
+                    ok = false;
+                    break;
+                }
             }
             if (!ok) break;
-            // ---- epilogue: partial state of this row for this item ----
-            // Every thread waits for the item's O before it frees it, so
-            // arrivals of one item never land in an earlier item's phase.
-            if (!__all_sync(0xffffffffu,
-                            tc::mbar_wait(bar(Bb::ODONE), uint32_t(k) & 1u, s_abort, P.err, kErrWaitSoftmax)))
+            // an item with no block has nothing to overlap with
+            if (pend && !epilogue()) {
+                ok = false;
                 break;
-            tc::tc_fence_after();
-            const int orow = seq * P.Hq + it.h * P.G + row % P.G;
-            const size_t idx = size_t(it.split) * P.B * P.Hq + size_t(orow);
-            float* xb = xl + (k & 1) * (2 * kRows);
-            if (it.nblk > 0) {
-                if (rows) {
-                    // Each thread holds its row's half of O.  Stores of one
-                    // value per thread would touch 32 rows (lines) per
-                    // instruction, so the warp stages 16 columns of its 32
-                    // rows at a time in shared memory and stores them as 8
-                    // rows x 64 contiguous bytes per instruction (16-byte
-                    // units rotated by row pair, so neither side conflicts).
-                    // (a partial-state index fits in 32 bits: the workspace holds 16 x
-                    // rows x 520 bytes, far below 2^31 rows of device memory)
-                    const int my_idx = valid ? int(idx) : -1;
-                    int ridx[4];
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) ridx[i] = __shfl_sync(0xffffffffu, my_idx, i * 8 + lane / 4);
-                    float* stg = reinterpret_cast<float*>(smem + C::OFF_STG + (warp - 4) * C::STG_BYTES);
-                    const int u = lane & 3;
-#pragma unroll
-                    for (int q = 0; q < C::OCH / 32; ++q) {
-                        float v[32];
-                        tc::tmem_ld32(tmem + lane_base + C::COL_O + wg * C::OCH + q * 32, v);
-                        tc::tmem_wait_ld();
-#pragma unroll
-                        for (int h = 0; h < 2; ++h) {
-#pragma unroll
-                            for (int w = 0; w < 4; ++w) {
-                                const int slot = (w + (lane >> 1)) & 3;
-                                *reinterpret_cast<float4*>(stg + lane * 16 + slot * 4) =
-                                    make_float4(v[h * 16 + w * 4], v[h * 16 + w * 4 + 1], v[h * 16 + w * 4 + 2],
-                                                v[h * 16 + w * 4 + 3]);
-                            }
-                            __syncwarp();
-#pragma unroll
-                            for (int i = 0; i < 4; ++i) {
-                                const int r = i * 8 + lane / 4;
-                                const float4 x =
-                                    *reinterpret_cast<const float4*>(stg + r * 16 + ((u + (r >> 1)) & 3) * 4);
-                                if (ridx[i] >= 0)
-                                    *reinterpret_cast<float4*>(P.ws_o + size_t(ridx[i]) * D + wg * C::OCH + q * 32 +
-                                                               h * 16 + u * 4) = x;
-                            }
-                            __syncwarp();
-                        }
-                    }
-                }
-                // a row's sum: its segments' sums in key order, then the two
-                // halves
-                xb[wg * kRows + row] = l_seg0 + l_seg1;
-                tc::mbar_arrive(bar(Bb::LXCH));
-                if (!__all_sync(0xffffffffu,
-                                tc::mbar_wait(bar(Bb::LXCH), uint32_t(k) & 1u, s_abort, P.err, kErrWaitSoftmax)))
-                    break;
-                if (wg == 0 && valid) P.ws_ml[idx] = make_float2(m_run, xb[row] + xb[kRows + row]);
-            } else {
-                // an empty split: a state with no keys (still one exchange
-                // round, so every item moves the exchange barrier once)
-                tc::mbar_arrive(bar(Bb::LXCH));
-                if (!__all_sync(0xffffffffu,
-                                tc::mbar_wait(bar(Bb::LXCH), uint32_t(k) & 1u, s_abort, P.err, kErrWaitSoftmax)))
-                    break;
-                if (wg == 0 && valid) P.ws_ml[idx] = make_float2(-INFINITY, 0.f);
             }
-            tc::tc_fence_before();
-            tc::mbar_arrive(bar(Bb::OFREE));
+            // ---- this item's partial state: written after the next item's
+            // first block ----
+            const int orow = seq * P.Hq + it.h * P.G + row % P.G;
+            // (a partial-state index fits in 32 bits: the workspace holds 16 x
+            // rows x 520 bytes, far below 2^31 rows of device memory)
+            pend_idx = valid ? int(size_t(it.split) * P.B * P.Hq + size_t(orow)) : -1;
+            pend_full = it.nblk > 0;
+            pend_rows = rows;
+            pend_k = k;
+            // a row's sum: its segments' sums in key order, then (in the
+            // epilogue) the two halves
+            pend_m = m_run;
+            pend_l = l_seg0 + l_seg1;
+            pend = true;
+            if (!kDefer && !epilogue()) {
+                ok = false;
+                break;
+            }
         }
+        if (ok && pend) epilogue();
     }
     tc::tc_fence_before();
     __syncthreads();
