@@ -59,8 +59,8 @@ NOMINAL_HBM_GBS = 8000.0
 # reduced ladder case (read + written bytes / algorithmic bytes of that launch);
 # traffic grows in proportion to the units a launch processes.  Only kernels
 # whose current build was captured are listed.
-TRAFFIC_PER_ALGORITHMIC_BYTE = {"generated_span_pass": (539.056 + 5.854) / 541.065,
-                                "prompt_span_pass": (236.987 + 4.719) / 234.881}
+TRAFFIC_PER_ALGORITHMIC_BYTE = {"generated_span_pass": (539.052 + 5.846) / 541.065,
+                                "prompt_span_pass": (237.009 + 4.820) / 234.881}
 
 
 def step_schedule(T: int, n: int, offset: int = 0):
