@@ -449,7 +449,8 @@ splice_status attn_common(splice_desc* d, int layer, int step, const splice_bf16
     // waits for whatever precedes it on the stream before it reads anything,
     // then lets the second pass launch; the second pass's CTAs take the SMs
     // the first pass's CTAs leave, and it waits for the first pass before it
-    // exits; the merge is queued behind the second pass.  So the first pass's
+    // exits; the merge is queued behind the second pass (unless the
+    // generated-span pass merges every row, p.gs_merge below).  So the first pass's
     // tail is filled and the second pass's is not.  The generated-span pass
     // goes first when the prompt-span pass holds at least
     // kPrefixFirstKeysPerSm keys per SM: then the prompt-span pass's items
