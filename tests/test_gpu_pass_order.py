@@ -98,6 +98,28 @@ def test_pass_order_other_head_dims(name, points):
     sb.close()
 
 
+def test_prompt_span_first_launches_no_merge():
+    """With the prompt-span pass first and one split of each span, the
+    generated-span pass merges every row and the call launches two kernels;
+    with the generated-span pass first the merge kernel is launched too.
+    The outputs are the same bits either way (checked above)."""
+    wl = WL.get("qwen3-4b")
+    sb = SweepBatch(wl, 0)
+    l, t = 5, 40
+    sb.gen_inputs(l, t)
+    counts = {}
+    for order in (1, 2):
+        S.splice_debug_pass_order(sb.desc, order)
+        before = S.splice_kernel_launches(sb.desc)
+        sb.step(l, t)
+        torch.cuda.synchronize()
+        counts[order] = S.splice_kernel_launches(sb.desc) - before
+    S.splice_debug_pass_order(sb.desc, 0)
+    S.splice_check_device_error(sb.desc)
+    assert counts == {1: 2, 2: 3}, counts
+    sb.close()
+
+
 def test_pass_order_rejects_bad_value():
     wl = WL.get("tiny")
     sb = SweepBatch(wl, 0)
