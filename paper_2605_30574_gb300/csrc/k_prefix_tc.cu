@@ -23,7 +23,8 @@
 //                 P (bf16) over their own half of the slot in TMEM, rescale
 //                 their half of O when the reference moves, and at the item's
 //                 end write the row's partial state (m, l, o) to the
-//                 workspace.  Warps whose 32 rows are all past the tile's end
+//                 workspace, through a per-warp staging buffer so the stores
+//                 leave in row-contiguous pieces.  Warps whose 32 rows are all past the tile's end
 //                 skip the arithmetic but keep every barrier.
 //   warp 3        P V issuer (one elected lane): O += P V with P read from
 //                 TMEM as soon as the softmax has written it -- a separate
@@ -34,8 +35,9 @@
 // positions (a per-row bitmask), and items over the slot's encoded rows (a
 // store of their own, split like a span) give the rest of the donor span.
 //
-// The merge kernel combines these partials with those of the generated span
-// (and the ZERO closed form).  Every wait is bounded: a wait that runs out
+// The merge kernel (or, with this pass first and one split of each span, the
+// generated-span pass) combines these partials with those of the generated
+// span (and the ZERO closed form).  Every wait is bounded: a wait that runs out
 // sets a CTA abort flag and an error bit in the descriptor's error word; all
 // roles then leave their loops, outstanding copies and MMAs are waited for
 // (bounded), TMEM is freed and the CTA exits.

@@ -7,7 +7,8 @@
 //     split) and, inside an item, blocks of 16 keys: a fixed stream per warp
 //     when this pass goes first, items claimed at run time (one ahead) when
 //     it runs behind the prompt-span pass, so warps that start late (on SMs
-//     that pass still holds) simply take fewer;
+//     that pass still holds) simply take fewer; the issue cursor decodes
+//     each item once and hands it to the consumer through a per-warp ring;
 //   * every block's K and V rows (contiguous in the generated-span store) are
 //     fetched by one bulk async copy (cp.async.bulk, mbarrier-tracked) into a
 //     two-stage per-warp ring; the next block -- of this item or the next one
@@ -23,8 +24,11 @@
 //     logits and the row sums are reduced once per item;
 //   * packed fp32x2 FMAs (FFMA2) for both q . k and p . v;
 //   * online softmax with a lazily moved reference max: the common path
-//     needs no rescale and no cross-lane max.
-// Emits the partial state (m, l, o) of every row, like the prompt-span pass.
+//     needs no rescale and no cross-lane max; at an item's end the key
+//     groups' states are combined by a reduce-scatter.
+// Emits the partial state (m, l, o) of every row, like the prompt-span pass
+// -- or, behind the prompt-span pass with one split of each span, merges
+// the rows itself and writes the output (no merge kernel then).
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
